@@ -1,0 +1,208 @@
+/*
+ * gefen.h -- C ABI of libgefen.so, the GB300 (sm_103a) implementation of the
+ * hot path of the Gefen optimizer (arXiv 2606.13894, "Gefen: Optimized
+ * Stochastic Optimizer").
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ *  - Plain C types only.  Device pointers point to CUDA global memory of the
+ *    current device; "host" pointers to ordinary host memory.  bf16 values are
+ *    passed as their uint16_t bit patterns.
+ *  - The caller owns every buffer.  The library never allocates device memory:
+ *    scratch comes from a caller-provided workspace whose size the matching
+ *    *_workspace_size() call returns (0 means none is needed; a NULL workspace
+ *    is then allowed).  Calls keep no state between invocations.
+ *  - All work is enqueued on `stream` (a cudaStream_t; NULL is the legacy
+ *    default stream) and returns without waiting, unless a call's description
+ *    says it synchronises.
+ *  - Arguments are validated on the host before anything is enqueued; a bad
+ *    argument returns GEFEN_EINVAL (or GEFEN_ENOMEM for a short workspace) and
+ *    leaves every buffer untouched.  A failed launch returns GEFEN_ECUDA.  A
+ *    fault that happens later on the device surfaces from the next CUDA call
+ *    or from gefen_sync_status().
+ *  - Calls on different streams that write the same buffers race; the library
+ *    does not order them.
+ */
+#ifndef GEFEN_H
+#define GEFEN_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* gefen_stream_t; /* same type as cudaStream_t */
+
+typedef enum {
+    GEFEN_OK = 0,
+    GEFEN_EINVAL = 1,       /* bad argument (host-side check, nothing enqueued) */
+    GEFEN_ECUDA = 2,        /* a CUDA runtime call or kernel launch failed */
+    GEFEN_ENOMEM = 3,       /* workspace smaller than the size query requires */
+    GEFEN_ETIMEOUT = 4,     /* reserved: a bounded device wait expired */
+    GEFEN_EUNSUPPORTED = 5, /* not an sm_103 device, or a size past a stated limit */
+    GEFEN_EDEVICE = 6       /* the device-side check of a call's data failed */
+} gefen_status_t;
+
+/* One parameter tensor inside the flat arenas of gefen_step().
+ * Its elements are params[offset .. offset+numel) (likewise grads and codes);
+ * its blocks are the consecutive runs [offset + b*period, offset + (b+1)*period)
+ * for b = 0 .. numel/period - 1 (Algorithm 2 reshapes the flattened tensor into
+ * (n/p) x p), and block b's state is v[block_offset + b], scale[block_offset + b].
+ * Requirements: offset % 16 == 0, numel >= 0, period >= 1, numel % period == 0;
+ * element ranges of different tensors do not overlap, nor do block ranges. */
+typedef struct {
+    int64_t offset;
+    int64_t numel;
+    int64_t period;
+    int64_t block_offset;
+} gefen_tensor_t;
+
+/* Hyperparameters of Algorithm 1 (AdamW's: stepsize alpha = lr, weight decay
+ * lambda, decay rates beta1, beta2 in [0,1), eps) and the step counter t >= 1
+ * used by both bias corrections.  flags: see GEFEN_HIST*. */
+typedef struct {
+    double lr;
+    double beta1;
+    double beta2;
+    double eps;
+    double weight_decay;
+    int64_t step;
+    uint32_t flags;
+} gefen_hparams_t;
+
+/* Also histogram x_i = m_i / s'_b of every element of every block with
+ * s'_b > 0 into `hist` during the step (the input of a codebook refit). */
+#define GEFEN_HIST 1u
+/* Only histogram g_i / max_{j in block}|g_j| of every nonzero block and write
+ * nothing else: the histogram of Algorithm 3 built from the first gradient. */
+#define GEFEN_HIST_GRAD_ONLY 2u
+
+/* Largest histogram supported by every call (bins), and largest codebook. */
+#define GEFEN_MAX_BINS 65536
+#define GEFEN_MAX_LEVELS 256
+
+/* Text for a status code (static storage). */
+const char* gefen_status_string(gefen_status_t s);
+
+/* Waits for `stream`, then reports a pending CUDA error as GEFEN_ECUDA. */
+gefen_status_t gefen_sync_status(gefen_stream_t stream);
+
+/* -------------------------------------------------------------------------
+ * gefen_step -- one iteration of Algorithm 1's loop body for every tensor.
+ *
+ * For each block b of each tensor, with codes c_i, scale s_b, shared v_b:
+ *   m_i  = beta1 * codebook_dec[c_i] * s_b + (1 - beta1) * g_i
+ *   s'_b = max_i |m_i|                                      (Quantize, absmax)
+ *   v_b  = beta2 * v_b + (1 - beta2) * mean_i g_i^2         (one v per block)
+ *   theta_i -= lr * ( m_i/(1-beta1^t) / (sqrt(v_b/(1-beta2^t)) + eps)
+ *                     + weight_decay * theta_i )
+ *   c_i  = index of the level of codebook_enc nearest to m_i / s'_b (ties to
+ *          the lower index); s_b = s'_b.
+ * The update uses the unquantised m_i.  A block with s'_b = 0 stores the level
+ * nearest to 0 in every c_i.  Initial state (Algorithm 1, "m_0 <- 0",
+ * "v_0 <- 0"): codes at the level nearest 0, scale = 0, v = 0.  After a
+ * codebook refit, pass the old codebook as codebook_dec and the new one as
+ * codebook_enc for one step.
+ *
+ * params  f32[*]  device, in/out     grads  bf16[*] device, in
+ * codes   u8[*]   device, in/out     v, scale f32[*] device, in/out (per block)
+ * codebook_dec, codebook_enc  f32[k] device, sorted ascending, 2 <= k <= 256
+ * hist    u64[hist_bins] device, counts are ADDED (caller zeroes); required
+ *         when a GEFEN_HIST* flag is set, else ignored (may be NULL).
+ *         1 <= hist_bins <= GEFEN_MAX_BINS.  Cell i of B is
+ *         [-1 + 2i/B, -1 + 2(i+1)/B), +1 in the last (fp32 arithmetic).
+ * params, grads, codes must be 16-byte aligned.  With GEFEN_HIST_GRAD_ONLY
+ * only grads, hist and the tensor table are used.
+ * workspace: gefen_step_workspace_size() bytes, 256-byte aligned.
+ * ------------------------------------------------------------------------- */
+size_t gefen_step_workspace_size(const gefen_tensor_t* tensors, int32_t ntensors,
+                                 uint32_t flags);
+gefen_status_t gefen_step(const gefen_tensor_t* tensors, int32_t ntensors,
+                          float* params, const uint16_t* grads, uint8_t* codes,
+                          float* v, float* scale, const float* codebook_dec,
+                          const float* codebook_enc, int32_t k,
+                          gefen_hparams_t hp, uint64_t* hist, int32_t hist_bins,
+                          void* workspace, size_t workspace_bytes,
+                          gefen_stream_t stream);
+
+/* -------------------------------------------------------------------------
+ * gefen_refit_codebook -- Algorithm 3 (Exact DP Quantization Codebook
+ * Learning) with Appendix D's interval costs.
+ *
+ * Input: either n fp32 values x (device; each counted in the cell above, NaN
+ * in none) or, when x == NULL, a histogram hist_in u64[bins] (device).
+ * The nonempty cells j = 1..b (ascending, centre u_j/bins with the odd integer
+ * u_j = 2*i_j + 1 - bins) are split into k contiguous runs minimising the
+ * squared error with the first level fixed at -1, the last at +1 and every
+ * other level at its run's count-weighted mean; every level gets >= 1
+ * nonempty cell.  Costs use exact integer moments:
+ *   interior run:  (double)(s0*s2 - s1^2) / (double)s0
+ *   first level:   (double)(s2 + 2B*s1 + B^2*s0),  last: (double)(s2 - 2B*s1 + B^2*s0)
+ * (round-to-nearest double, units of 1/B^2), D[r][k'] = min over the run
+ * start l of D[l-1][k'-1] + cost, ties to the smallest l.  The result equals
+ * the full O(b^2 k) scan bit for bit.  With b < k nonempty cells the DP runs
+ * with b levels and the codebook is padded with +1 (b <= 1: [-1,+1,+1,...]).
+ *
+ * codebook_out   f32[k] device: C[0] = -1, C[k_eff-1] = +1, interior levels
+ *                = (s1/s0)/bins rounded to fp32.
+ * hist_out       u64[bins] device, nullable: the histogram used.
+ * cell_start_out i32[k] device, nullable: first cell index of each level (-1
+ *                for padding).
+ * cost_out       f64[1] device, nullable: the optimum D[b][k_eff].
+ * Requirements: 1 <= bins <= GEFEN_MAX_BINS, 2 <= k <= GEFEN_MAX_LEVELS,
+ * n >= 0, x 16-byte aligned, total count N < 2^62 with N*(bins-1)^2 < 2^64
+ * (checked on the device: on
+ * failure the outputs are left untouched and gefen_refit_status() reports
+ * GEFEN_EDEVICE).  workspace: gefen_refit_workspace_size() bytes.
+ * ------------------------------------------------------------------------- */
+size_t gefen_refit_workspace_size(int32_t bins, int32_t k);
+gefen_status_t gefen_refit_codebook(const float* x, int64_t n, const uint64_t* hist_in,
+                                    int32_t bins, int32_t k, float* codebook_out,
+                                    uint64_t* hist_out, int32_t* cell_start_out,
+                                    double* cost_out, void* workspace,
+                                    size_t workspace_bytes, gefen_stream_t stream);
+
+/* Device-side status of the last gefen_refit_codebook() that used this
+ * workspace; synchronises `stream`.  k_eff_out (host, nullable) receives the
+ * number of levels the DP used. */
+gefen_status_t gefen_refit_status(const void* workspace, int32_t* k_eff_out,
+                                  gefen_stream_t stream);
+
+/* The full DP tables of the last refit in this workspace, for inspection:
+ * D (f64) and the minimising run start l (i32, 1-based; 0 where undefined),
+ * both (k+1) x (bins+1) row-major by level; entries the recurrence does not
+ * define are +inf / 0.  Copies device to device on `stream`. */
+gefen_status_t gefen_refit_tables(const void* workspace, int32_t bins, int32_t k,
+                                  double* dtable_out, int32_t* argl_out,
+                                  gefen_stream_t stream);
+
+/* -------------------------------------------------------------------------
+ * gefen_infer_blocks -- Algorithm 2 (Automatic Block Partitioning) for one
+ * flattened gradient tensor g (bf16 bits, device, numel elements).
+ *
+ * z_j = log(g_j^2 + eps).  For every divisor p of n (ascending):
+ *   mu_i(p) = mean of z over the i-th run of p elements,
+ *   S(p)    = mean over i of |mu_{i+1}(p) - mu_i(p)|      (S(n) undefined)
+ * (the partition-score equation of Sec. 5.1).  The period is the divisor
+ * 1 < p < n whose score is a strict local maximum over the sorted divisor list
+ * and is the largest such (smallest p on ties); 1 if there is none.
+ * Synchronises `stream` and writes period_out (host).  scores_out (host,
+ * nullable, scores_cap entries) receives S(p) for the divisors in ascending
+ * order; ndiv_out (host, nullable) the divisor count.  1 <= numel <= 2^32,
+ * eps > 0, grad 16-byte aligned.  A non-finite gradient returns GEFEN_EDEVICE.
+ * workspace: gefen_infer_workspace_size(numel) bytes.
+ * ------------------------------------------------------------------------- */
+size_t gefen_infer_workspace_size(int64_t numel);
+gefen_status_t gefen_infer_blocks(const uint16_t* grad, int64_t numel, double eps,
+                                  int64_t* period_out, double* scores_out,
+                                  int64_t scores_cap, int64_t* ndiv_out,
+                                  void* workspace, size_t workspace_bytes,
+                                  gefen_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GEFEN_H */

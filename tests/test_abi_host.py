@@ -1,0 +1,118 @@
+"""Host-side checks of the C ABI: the library builds and loads, exports every
+function include/gefen.h declares, and rejects bad arguments on the host
+(before any device work), so none of these calls needs a GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2606_13894_gb300 import gefen as G
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "gefen.h")
+
+
+def _declared():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(gefen_[a-z_0-9]+)\s*\(", src)))
+
+
+def test_every_declared_symbol_is_exported():
+    lib = G.load()
+    names = _declared()
+    assert len(names) >= 10
+    for n in names:
+        assert hasattr(lib, n), n
+    assert set(names) == set(G.EXPORTS)
+
+
+def test_status_strings():
+    assert G.gefen_status_string(0) == "ok"
+    assert "invalid" in G.gefen_status_string(1)
+    assert G.gefen_status_string(99) == "unknown status"
+
+
+def _table(entries):
+    return G.tensor_table(entries)
+
+
+def test_step_workspace_sizes_follow_the_plan():
+    # small blocks need no scratch; big blocks need per-chunk partials
+    assert G.gefen_step_workspace_size(_table([(0, 4096, 64, 0)])) == 0
+    big = G.gefen_step_workspace_size(_table([(0, 1 << 20, 1 << 20, 0)]))
+    assert big > 0
+    hist = G.gefen_step_workspace_size(_table([(0, 4096, 64, 0)]), G.GEFEN_HIST)
+    assert hist >= 4096 * 4
+    # invalid tables report 0
+    assert G.gefen_step_workspace_size(_table([(0, 100, 7, 0)])) == 0
+    assert G.gefen_step_workspace_size(_table([(8, 64, 64, 0)])) == 0
+
+
+def test_refit_and_infer_workspace_sizes():
+    assert G.gefen_refit_workspace_size(4096, 256) > 257 * 4097 * 12
+    assert G.gefen_refit_workspace_size(0, 256) == 0
+    assert G.gefen_refit_workspace_size(65537, 256) == 0
+    assert G.gefen_refit_workspace_size(4096, 1) == 0
+    assert G.gefen_infer_workspace_size(1000) > 1001 * 16
+    assert G.gefen_infer_workspace_size(0) == 0
+
+
+def _hp(**kw):
+    d = dict(lr=1e-3, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=0.0, step=1, flags=0)
+    d.update(kw)
+    return G.gefen_hparams_t(d["lr"], d["beta1"], d["beta2"], d["eps"], d["weight_decay"], d["step"], d["flags"])
+
+
+FAKE = ctypes.c_void_p(1 << 20)  # 16-byte aligned, never dereferenced on these paths
+
+
+def _step(table, hp=None, k=256, params=FAKE, grads=FAKE, ws=None, ws_bytes=0, hist=None, bins=0):
+    arr, n = table
+    return G.load().gefen_step(arr, n, params, grads, FAKE, FAKE, FAKE, FAKE, FAKE, k, hp or _hp(),
+                               hist, bins, ws, ws_bytes, None)
+
+
+@pytest.mark.parametrize("entries", [
+    [(0, 100, 7, 0)],                 # period does not divide numel
+    [(8, 64, 64, 0)],                 # offset not a multiple of 16
+    [(0, 64, 0, 0)],                  # period 0
+    [(0, 64, 16, 0), (32, 64, 16, 8)],  # overlapping element ranges
+    [(0, 64, 16, 0), (64, 64, 16, 2)],  # overlapping block ranges
+    [(-16, 64, 16, 0)],               # negative offset
+])
+def test_step_rejects_bad_tables(entries):
+    assert _step(_table(entries)) == G.GEFEN_EINVAL
+
+
+def test_step_rejects_bad_scalars_and_pointers():
+    t = _table([(0, 64, 16, 0)])
+    assert _step(t, k=1) == G.GEFEN_EINVAL
+    assert _step(t, k=257) == G.GEFEN_EINVAL
+    assert _step(t, hp=_hp(step=0)) == G.GEFEN_EINVAL
+    assert _step(t, hp=_hp(beta1=1.0)) == G.GEFEN_EINVAL
+    assert _step(t, hp=_hp(beta2=-0.1)) == G.GEFEN_EINVAL
+    assert _step(t, hp=_hp(eps=float("nan"))) == G.GEFEN_EINVAL
+    assert _step(t, hp=_hp(flags=3)) == G.GEFEN_EINVAL
+    assert _step(t, hp=_hp(flags=8)) == G.GEFEN_EINVAL
+    assert _step(t, params=None) == G.GEFEN_EINVAL
+    assert _step(t, params=ctypes.c_void_p((1 << 20) + 4)) == G.GEFEN_EINVAL  # misaligned
+    assert _step(t, hp=_hp(flags=G.GEFEN_HIST)) == G.GEFEN_EINVAL             # hist missing
+    assert _step(t, hp=_hp(flags=G.GEFEN_HIST), hist=FAKE, bins=70000) == G.GEFEN_EINVAL
+    big = _table([(0, 1 << 20, 1 << 20, 0)])
+    assert _step(big) == G.GEFEN_ENOMEM  # scratch needed but none given
+
+
+def test_refit_and_infer_reject_bad_arguments():
+    L = G.load()
+    P = FAKE
+    assert L.gefen_refit_codebook(None, 0, None, 4096, 256, P, None, None, None, P, 1 << 30, None) == G.GEFEN_EINVAL
+    assert L.gefen_refit_codebook(P, 10, None, 4096, 1, P, None, None, None, P, 1 << 30, None) == G.GEFEN_EINVAL
+    assert L.gefen_refit_codebook(P, 10, None, 0, 256, P, None, None, None, P, 1 << 30, None) == G.GEFEN_EINVAL
+    assert L.gefen_refit_codebook(P, 10, None, 4096, 256, P, None, None, None, P, 16, None) == G.GEFEN_ENOMEM
+    per = ctypes.c_int64(0)
+    assert L.gefen_infer_blocks(P, 0, 1e-8, ctypes.byref(per), None, 0, None, P, 1 << 30, None) == G.GEFEN_EINVAL
+    assert L.gefen_infer_blocks(P, 64, 0.0, ctypes.byref(per), None, 0, None, P, 1 << 30, None) == G.GEFEN_EINVAL
+    assert L.gefen_infer_blocks(P, 64, 1e-8, None, None, 0, None, P, 1 << 30, None) == G.GEFEN_EINVAL
+    assert L.gefen_infer_blocks(P, 64, 1e-8, ctypes.byref(per), None, 0, None, P, 8, None) == G.GEFEN_ENOMEM
