@@ -37,7 +37,9 @@ WORKLOAD = "llama-1.5b"
 METRIC = "Gefen step throughput (Gparams/s)"
 UNIT = "Gparams/s"
 REFIT_EVERY = 10
-BINS = 65536
+BINS = 4096          # Algorithm 3: 16k cells with k = 256
+MICRO_BINS = 65536   # the refit micro-benchmark
+MICRO_N = 1_499_987_968  # 1.5e9 values rounded to whole blocks of 4096
 K = 256
 HP = dict(lr=1e-4, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=0.0)  # Appendix I, Llama
 SEED = 0
@@ -138,8 +140,10 @@ def launches_per_step(periods, flags_hist: bool) -> int:
     for p in periods:
         if p == 1:
             cls.add("p1")
+        elif p % 16 == 0 and p <= 4096:
+            cls.add("s4k")
         elif p % 16 == 0 and p <= 8192:
-            cls.add("t16v2")
+            cls.add("s8k")
         elif p % 16 == 0 and p <= 16384:
             cls.add("t16v4")
         elif p <= 2048:
@@ -148,6 +152,15 @@ def launches_per_step(periods, flags_hist: bool) -> int:
             big |= 1 if p % 16 == 0 else 2
     n = len(cls) + 3 * bin(big).count("1")
     return n + (1 if flags_hist else 0)
+
+
+def period_summary(specs, periods):
+    """Inferred period -> (tensors, params) over the workload."""
+    out = {}
+    for s, p in zip(specs, periods):
+        t, n = out.get(str(p), (0, 0))
+        out[str(p)] = (t + 1, n + s.numel)
+    return out
 
 
 # ----------------------------------------------------------------- GPU arm
@@ -262,6 +275,7 @@ def run_gpu(args, world, rank, local):
     torch.cuda.synchronize()
     time.sleep(0.05)
     ck = clocks.stop()
+    G.gefen_step_status(ws)  # raises if a bounded device wait gave up
     elapsed_ms = ev0.elapsed_time(ev1)
     if world > 1:
         import torch.distributed as dist
@@ -313,11 +327,40 @@ def run_gpu(args, world, rank, local):
                   "hist_step_ms": statistics.mean(refit_step_ms) if refit_step_ms else None,
                   "count": nref},
         "init": {"infer_blocks_s": infer_s, "first_codebook_s": init_codebook_s},
+        "periods": period_summary(specs, periods),
         "e2e": e2e, "gpu_launches": launches, "clocks": ck,
     }
+    if rank == 0 and not args.no_microbench:
+        res["refit_microbench"] = refit_microbench(G, synth, dev)
     if rank == 0 and not args.no_cpu_baseline:
         res["cpu_baseline"] = cpu_baseline(args)
     return res
+
+
+def refit_microbench(G, synth, dev):
+    """Histogram of 1.5e9 normalised values into 65536 cells, then the exact DP
+    to 256 levels; CUDA-event times of each part (after one untimed run)."""
+    x = synth.refit_values(MICRO_N, SEED + 7, device=dev)
+    hist = torch.zeros(MICRO_BINS, dtype=torch.int64, device=dev)
+    cb = torch.empty(K, dtype=torch.float32, device=dev)
+    ws = G.workspace(G.gefen_refit_workspace_size(MICRO_BINS, K), dev)
+    G.gefen_refit_codebook(bins=MICRO_BINS, k=K, codebook_out=cb, x=x, hist_out=hist, workspace_buf=ws)
+    torch.cuda.synchronize()
+    e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+    e[0].record()
+    G.gefen_refit_codebook(bins=MICRO_BINS, k=K, codebook_out=cb, x=x, hist_out=hist, workspace_buf=ws)
+    e[1].record()
+    G.gefen_refit_codebook(bins=MICRO_BINS, k=K, codebook_out=cb, hist_in=hist, workspace_buf=ws)
+    e[2].record()
+    torch.cuda.synchronize()
+    ke = G.gefen_refit_status(ws)
+    hist_dp_ms, dp_ms = e[0].elapsed_time(e[1]), e[1].elapsed_time(e[2])
+    del x
+    torch.cuda.empty_cache()
+    return {"values": MICRO_N, "bins": MICRO_BINS, "levels": K, "k_eff": ke,
+            "nonempty_cells": int((hist > 0).sum().item()),
+            "hist_ms": hist_dp_ms - dp_ms, "dp_ms": dp_ms, "total_ms": hist_dp_ms,
+            "hist_gbs": 4 * MICRO_N / ((hist_dp_ms - dp_ms) * 1e-3) / 1e9}
 
 
 def run_e2e(G, table, theta, codes, v, sc, cb, ws, gpool, nparams, stream, args, state, one_step_ctx):
@@ -439,6 +482,7 @@ def main():
     ap.add_argument("--cpu-params", type=int, default=20_000_000, help="params in the cpu_baseline sample")
     ap.add_argument("--ref-params", type=float, default=20e6, help="oracle params per reference step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-microbench", action="store_true", help="skip the 65536-cell refit measurement")
     args = ap.parse_args()
     world, rank, local = dist_env()
     if args.impl == "reference":

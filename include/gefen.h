@@ -115,7 +115,9 @@ gefen_status_t gefen_sync_status(gefen_stream_t stream);
  *         [-1 + 2i/B, -1 + 2(i+1)/B), +1 in the last (fp32 arithmetic).
  * params, grads, codes must be 16-byte aligned.  With GEFEN_HIST_GRAD_ONLY
  * only grads, hist and the tensor table are used.
- * workspace: gefen_step_workspace_size() bytes, 256-byte aligned.
+ * workspace: gefen_step_workspace_size() bytes (at least 256), 256-byte
+ * aligned; its first 256 bytes must be zero before the first call (they hold
+ * the flag gefen_step_status() reads).
  * ------------------------------------------------------------------------- */
 size_t gefen_step_workspace_size(const gefen_tensor_t* tensors, int32_t ntensors,
                                  uint32_t flags);
@@ -126,6 +128,11 @@ gefen_status_t gefen_step(const gefen_tensor_t* tensors, int32_t ntensors,
                           gefen_hparams_t hp, uint64_t* hist, int32_t hist_bins,
                           void* workspace, size_t workspace_bytes,
                           gefen_stream_t stream);
+
+/* Synchronises `stream` and reports whether a step that used this workspace
+ * gave up a bounded wait for its own shared-memory copies (GEFEN_ETIMEOUT; the
+ * step's outputs are then not valid).  Reading the flag clears it. */
+gefen_status_t gefen_step_status(void* workspace, gefen_stream_t stream);
 
 /* -------------------------------------------------------------------------
  * gefen_refit_codebook -- Algorithm 3 (Exact DP Quantization Codebook

@@ -8,18 +8,21 @@
 //   last      (double)(s2 - 2B s1 + B^2 s0)      (centre +1)
 // D[r][k'] = min_{k' <= l <= r} D[l-1][k'-1] + cost(l..r), ties to the smallest l.
 //
-// One launch per level, one thread per end position r.  Instead of evaluating
-// all O(r) candidates in fp64 (slow on this part), each candidate is screened
-// in fp32 from the exact 128-bit numerator: the screened value v32 is within
-// 4e-7 relative of the canonical value, so [v32(1-2^-20), v32(1+2^-20)]
-// brackets it.  Whole runs of candidates are excluded with two exact facts:
-// the interior cost of [l..r] does not increase as l grows (a subset has no
-// larger squared error) and D[.][k'-1] does not decrease along r (more cells
-// for the same levels never cost less).  So for l in [a, e]:
-//   value(l) >= D[a-1][k'-1] + cost(e..r),   and for l >= a: value(l) >= D[a-1].
-// Candidates that survive (typically a handful near the optimum) are evaluated
-// with the canonical fp64 formula; the minimum over them, with ties to the
-// smallest l, equals the full scan bit for bit.
+// One launch per level, one warp per end position r.  fp64 is slow on this
+// part, so candidates are screened in float-float arithmetic (a pair of fp32
+// values, about 2^-43 relative error): D[.][k'-1] is kept as a (hi, lo) pair
+// and each cost comes from its exact 128-bit integer numerator.  Whole runs of
+// candidates are excluded with two exact facts: the interior cost of [l..r]
+// does not increase as l grows (a subset has no larger squared error) and
+// D[.][k'-1] does not decrease along r (more cells for the same levels never
+// cost less).  So for l in [a, e]:  value(l) >= D[a-1][k'-1] + cost(e..r).
+// A 32-wide window around a hint (the previous level's split at r, moved by
+// its share of the last cell) gives the best screened value u, one candidate
+// per lane; the rest of [k', r] is searched by 32-way subdivision (one run
+// bound per lane), dropping every run whose bound exceeds u by more than 2^-34
+// relative.  Survivors (near-ties only) get the
+// canonical fp64 value; their minimum, ties to the smallest l, equals the full
+// scan bit for bit.
 #include <algorithm>
 #include <cmath>
 
@@ -30,9 +33,10 @@ namespace gefen {
 
 namespace {
 
-constexpr int kDpThreads = 128;
-constexpr float kMLo = 1.0f - 9.5367431640625e-07f;  // 1 - 2^-20
-constexpr float kMHi = 1.0f + 9.5367431640625e-07f;  // 1 + 2^-20
+constexpr int kDpThreads = 64;
+constexpr float kEps = 5.820766091346741e-11f;  // 2^-34: exclusion margin (screen error < 2^-41)
+constexpr int kWin = 16;                         // window around the hint
+constexpr int kLeaf = 8;                         // runs this short are screened one by one
 
 struct Header {
     int32_t status;  // 0 ok, 1 moment overflow (N (B-1)^2 >= 2^64)
@@ -50,7 +54,7 @@ struct DpWs {
     uint64_t* P2;
     double* D;     // (k+1) x (B+1)
     int32_t* A;    // (k+1) x (B+1)
-    float* E;      // 2 x (B+2): E[l] = float(D[level][l-1]) for the next level
+    float2* E;     // 2 x (B+2): E[l] = (hi, lo) of D[level][l-1] for the next level
 };
 
 struct DpLayout {
@@ -71,7 +75,7 @@ DpLayout dp_layout(int B, int k) {
     L.P2 = o;  o += align_up(n1 * sizeof(uint64_t));
     L.D = o;   o += align_up(static_cast<size_t>(k + 1) * n1 * sizeof(double));
     L.A = o;   o += align_up(static_cast<size_t>(k + 1) * n1 * sizeof(int32_t));
-    L.E = o;   o += align_up(2 * (n1 + 1) * sizeof(float));
+    L.E = o;   o += align_up(2 * (n1 + 1) * sizeof(float2));
     L.total = o;
     return L;
 }
@@ -87,7 +91,7 @@ DpWs dp_ws(void* base, int B, int k) {
     w.P2 = reinterpret_cast<uint64_t*>(p + L.P2);
     w.D = reinterpret_cast<double*>(p + L.D);
     w.A = reinterpret_cast<int32_t*>(p + L.A);
-    w.E = reinterpret_cast<float*>(p + L.E);
+    w.E = reinterpret_cast<float2*>(p + L.E);
     return w;
 }
 
@@ -122,8 +126,76 @@ __device__ __forceinline__ Run run_of(const DpWs& W, int l, uint64_t P0r, int64_
     return q;
 }
 
-__device__ __forceinline__ float cost32_interior(const Run& q) {
-    return u128_to_float_approx(interior_num(q.s0, q.s1, q.s2)) * __frcp_rn(__ull2float_rn(q.s0));
+// ---------------------------------------------------- float-float values
+struct ff {
+    float hi, lo;
+};
+
+__device__ __forceinline__ ff ff_quick(float a, float b) {  // |a| >= |b|
+    const float s = __fadd_rn(a, b);
+    return ff{s, __fsub_rn(b, __fsub_rn(s, a))};
+}
+__device__ __forceinline__ ff ff_add(ff x, ff y) {
+    const float s = __fadd_rn(x.hi, y.hi);
+    const float bb = __fsub_rn(s, x.hi);
+    const float e = __fadd_rn(__fsub_rn(x.hi, __fsub_rn(s, bb)), __fsub_rn(y.hi, bb));
+    return ff_quick(s, __fadd_rn(e, __fadd_rn(x.lo, y.lo)));
+}
+__device__ __forceinline__ ff ff_sub(ff x, ff y) { return ff_add(x, ff{-y.hi, -y.lo}); }
+// n / d: one reciprocal, an exact product error by fma, one correction.
+__device__ __forceinline__ ff ff_div(ff n, ff d) {
+    const float r = __frcp_rn(d.hi);
+    const float q1 = __fmul_rn(n.hi, r);
+    const float p = __fmul_rn(q1, d.hi);
+    const float pe = __fmaf_rn(q1, d.hi, -p);
+    float rem = __fsub_rn(n.hi, p);
+    rem = __fsub_rn(rem, pe);
+    rem = __fadd_rn(rem, n.lo);
+    rem = __fsub_rn(rem, __fmul_rn(q1, d.lo));
+    return ff_quick(q1, __fmul_rn(rem, r));
+}
+// An unsigned 128-bit integer as hi + lo (top 64 bits kept: error < 2^-47).
+// Built from bit fields and 32-bit conversions only: 64-bit integer to float
+// conversions would run on the slow fp64 pipe of this part.
+__device__ __forceinline__ ff u128_to_ff(u128 v) {
+    uint64_t T;
+    int e2;  // value = T * 2^e2
+    if (v.hi) {
+        const int sh = __clzll(static_cast<long long>(v.hi));
+        T = sh ? (v.hi << sh) | (v.lo >> (64 - sh)) : v.hi;
+        e2 = 64 - sh;
+    } else if (v.lo) {
+        const int sh = __clzll(static_cast<long long>(v.lo));
+        T = v.lo << sh;
+        e2 = -sh;
+    } else {
+        return ff{0.0f, 0.0f};
+    }
+    // hi: the top 24 bits exactly (T has bit 63 set)
+    const uint32_t mant = static_cast<uint32_t>(T >> 40) & 0x7FFFFFu;
+    const float hi = __int_as_float(((127 + 63 + e2) << 23) | static_cast<int>(mant));
+    // lo: the remaining 40 bits, rounded once
+    const uint64_t R = T & 0xFFFFFFFFFFull;
+    const float r = __fmaf_rn(__uint2float_rn(static_cast<uint32_t>(R >> 32)), 4294967296.0f,
+                              __uint2float_rn(static_cast<uint32_t>(R)));
+    return ff_quick(hi, r * __int_as_float((127 + e2) << 23));
+}
+__device__ __forceinline__ ff d_to_ff(double d) {
+    if (isinf(d)) return ff{static_cast<float>(d), 0.0f};
+    const float hi = __double2float_rn(d);
+    return ff{hi, __double2float_rn(__dsub_rn(d, static_cast<double>(hi)))};
+}
+__device__ __forceinline__ ff cost_ff_interior(const Run& q) {
+    return ff_div(u128_to_ff(interior_num(q.s0, q.s1, q.s2)), u128_to_ff(u128{0ull, q.s0}));
+}
+// Whether every value bounded below by lb is certainly above the best
+// screened value u (margin 2^-34 relative, far above the screening error).
+__device__ __forceinline__ bool excluded(ff lb, ff u) {
+    return ff_sub(lb, u).hi > kEps * (lb.hi + u.hi);
+}
+__device__ __forceinline__ ff ld_ff(const float2* E, int l) {
+    const float2 e = E[l];
+    return ff{e.x, e.y};
 }
 
 __device__ __forceinline__ double cost64_interior(const Run& q) {
@@ -229,7 +301,8 @@ __global__ void __launch_bounds__(kDpThreads) k_dp_level1(int B, DpWs W) {
         W.D[n1 + r] = d;
         W.A[n1 + r] = (r >= 1 && r <= h.b) ? 1 : 0;
     }
-    W.E[1 * (n1 + 1) + g] = __double2float_rn(d);  // row 1 of the rolling E buffer
+    const ff e = d_to_ff(d);
+    W.E[1 * (n1 + 1) + g] = make_float2(e.hi, e.lo);  // row 1 of the rolling E buffer
 }
 
 // Candidate screen + canonical evaluation for one (r, level) -- interior.
@@ -242,134 +315,147 @@ __device__ __forceinline__ void take(Best& b, double v, int l) {
     if (v < b.v || (v == b.v && l < b.l)) { b.v = v; b.l = l; }
 }
 
-__device__ __forceinline__ Best search_interior(const DpWs& W, const double* __restrict__ Dp,
-                                                const float* __restrict__ Ep, int kk, int r, int hint) {
-    const uint64_t P0r = W.P0[r], P2r = W.P2[r];
-    const int64_t P1r = W.P1[r];
-    float best_hi = INFINITY;
+// Lexicographic (hi, lo) minimum over the warp.
+__device__ __forceinline__ ff warp_min_ff(ff v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float oh = __shfl_xor_sync(0xffffffffu, v.hi, o);
+        const float ol = __shfl_xor_sync(0xffffffffu, v.lo, o);
+        if (oh < v.hi || (oh == v.hi && ol < v.lo)) v = ff{oh, ol};
+    }
+    return v;
+}
+__device__ __forceinline__ Best warp_min_best(Best b) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const double ov = __shfl_xor_sync(0xffffffffu, b.v, o);
+        const int ol = __shfl_xor_sync(0xffffffffu, b.l, o);
+        take(b, ov, ol);
+    }
+    return b;
+}
+
+constexpr int kDpWarps = 8;      // warps (end positions) per CTA
+constexpr int kStackCap = 192;   // runs pending per warp
+
+// Everything one warp needs to screen and evaluate candidates for one r.
+struct RowCtx {
+    const DpWs* W;
+    const double* Dp;
+    const float2* Ep;
+    uint64_t P0r, P2r;
+    int64_t P1r;
+    int B, r;
+    bool last;  // +1-centred cost of the last level
+};
+
+// Screened value of the run [l..r] as the last cell (value of candidate l).
+__device__ __forceinline__ ff run_cost_ff(const RowCtx& c, int l) {
+    const Run q = run_of(*c.W, l, c.P0r, c.P1r, c.P2r);
+    return c.last ? u128_to_ff(fixed_num(q.s0, q.s1, q.s2, c.B, -1)) : cost_ff_interior(q);
+}
+__device__ __forceinline__ double run_cost_64(const RowCtx& c, int l) {
+    const Run q = run_of(*c.W, l, c.P0r, c.P1r, c.P2r);
+    return c.last ? u128_to_double_rn(fixed_num(q.s0, q.s1, q.s2, c.B, -1)) : cost64_interior(q);
+}
+
+// One round over up to 32 consecutive candidates [a, a+31] ∩ [a, e].
+__device__ __forceinline__ void eval_candidates(const RowCtx& c, int a, int e, int lane, ff& u, Best& bst) {
+    const int l = a + lane;
+    const bool in = l <= e;
+    ff v{INFINITY, 0.0f};
+    if (in) v = ff_add(ld_ff(c.Ep, l), run_cost_ff(c, l));
+    const ff vm = warp_min_ff(v);
+    if (vm.hi < u.hi || (vm.hi == u.hi && vm.lo < u.lo)) u = vm;
+    if (in && !excluded(v, u)) take(bst, __dadd_rn(c.Dp[l - 1], run_cost_64(c, l)), l);
+}
+
+__device__ Best search_row(const RowCtx& c, int kk, int hint, int lane, int2* stack) {
     Best bst{INFINITY, 0};
-    // 1. a window of 32 candidates around the hint
+    ff u{INFINITY, 0.0f};
+    const int r = c.r;
     int w0 = max(kk, hint - 8);
     const int w1 = min(r, w0 + 31);
     w0 = max(kk, w1 - 31);
-    for (int l = w0; l <= w1; ++l) {
-        const float v = __ldg(Ep + l) + cost32_interior(run_of(W, l, P0r, P1r, P2r));
-        best_hi = fminf(best_hi, v * kMHi);
+    eval_candidates(c, w0, w1, lane, u, bst);
+    int sp = 0;  // warp-uniform
+    if (lane == 0) {
+        if (w1 < r) stack[sp] = make_int2(w1 + 1, r);
+        if (w0 > kk) stack[sp + (w1 < r ? 1 : 0)] = make_int2(kk, w0 - 1);
     }
-    auto eval = [&](int l) {
-        const Run q = run_of(W, l, P0r, P1r, P2r);
-        const float v = __ldg(Ep + l) + cost32_interior(q);
-        best_hi = fminf(best_hi, v * kMHi);
-        if (v * kMLo <= best_hi) take(bst, __dadd_rn(__ldg(Dp + l - 1), cost64_interior(q)), l);
-    };
-    for (int l = w0; l <= w1; ++l) eval(l);
-    // 2. runs of 32 to the left: stop once even the smallest D plus the cost of
-    //    [e..r] exceeds the best (it only grows leftwards)
-    const float e_min = __ldg(Ep + kk);
-    for (int e = w0 - 1; e >= kk;) {
-        const int a = max(kk, e - 31);
-        const float ce = cost32_interior(run_of(W, e, P0r, P1r, P2r));
-        if ((e_min + ce) * kMLo > best_hi) break;
-        if ((__ldg(Ep + a) + ce) * kMLo <= best_hi)
-            for (int l = e; l >= a; --l) eval(l);
-        e = a - 1;
+    sp = (w1 < r ? 1 : 0) + (w0 > kk ? 1 : 0);
+    __syncwarp();
+    while (sp > 0) {
+        const int2 run = stack[--sp];
+        __syncwarp();
+        const int a = run.x, e = run.y, width = e - a + 1;
+        if (width <= 32) {
+            eval_candidates(c, a, e, lane, u, bst);
+            continue;
+        }
+        // 32 sub-runs; lane i bounds [ca, ce] by D[ca-1] + cost(ce..r)
+        const int cw = (width + 31) >> 5;
+        const int ca = a + lane * cw, ce = min(e, ca + cw - 1);
+        bool keep = false;
+        if (ca <= e) keep = !excluded(ff_add(ld_ff(c.Ep, ca), run_cost_ff(c, ce)), u);
+        const unsigned mask = __ballot_sync(0xffffffffu, keep);
+        const int cnt = __popc(mask);
+        if (sp + cnt > kStackCap) {
+            // no room to split: screen the run directly (never expected)
+            for (int b = a; b <= e; b += 32) eval_candidates(c, b, min(e, b + 31), lane, u, bst);
+            continue;
+        }
+        // nearest the window on top: left of the window -> highest sub-run last
+        const int below = __popc(mask & ((1u << lane) - 1u));
+        const int pos = (e < w0) ? below : (cnt - 1 - below);
+        if (keep) stack[sp + pos] = make_int2(ca, ce);
+        sp += cnt;
+        __syncwarp();
     }
-    // 3. runs of 32 to the right: stop once D alone exceeds the best
-    for (int a = w1 + 1; a <= r;) {
-        const float ea = __ldg(Ep + a);
-        if (ea * kMLo > best_hi) break;
-        const int e = min(r, a + 31);
-        const float ce = cost32_interior(run_of(W, e, P0r, P1r, P2r));
-        if ((ea + ce) * kMLo <= best_hi)
-            for (int l = a; l <= e; ++l) eval(l);
-        a = e + 1;
-    }
-    return bst;
+    return warp_min_best(bst);
 }
 
-// Interior level kk (2 <= kk < k_eff), or the last level kk == k_eff (only
-// r = b, scanned by CTA 0), or nothing (kk > k_eff).  Thread g covers r = g-1.
-__global__ void __launch_bounds__(kDpThreads) k_dp_level(int B, int kk, DpWs W) {
+// Level kk: interior (2 <= kk < k_eff) for every r, or the last level
+// (kk == k_eff) for r = b only, or nothing defined (kk > k_eff).  One warp per
+// r in [0, B]; every D[kk][r] is written (+inf where undefined).
+__global__ void __launch_bounds__(kDpWarps * 32) k_dp_level(int B, int kk, DpWs W) {
+    __shared__ int2 s_stack[kDpWarps][kStackCap];
     const Header h = *W.hdr;
     if (h.status) return;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int r = blockIdx.x * kDpWarps + warp;
+    if (r > B) return;
     const int n1 = B + 1;
-    const int g = blockIdx.x * blockDim.x + threadIdx.x;
-    const int r = g - 1;
-    const double* Dp = W.D + static_cast<size_t>(kk - 1) * n1;
-    const float* Ep = W.E + static_cast<size_t>((kk - 1) & 1) * (n1 + 1);
-    float* En = W.E + static_cast<size_t>(kk & 1) * (n1 + 1);
-    double* Dk = W.D + static_cast<size_t>(kk) * n1;
-    int32_t* Ak = W.A + static_cast<size_t>(kk) * n1;
-
-    if (kk == h.k_eff) {
-        // Last level (centre +1): one r = b, candidates split over CTA 0.
-        if (blockIdx.x == 0) {
-            __shared__ float s_hi[kDpThreads];
-            __shared__ double s_v[kDpThreads];
-            __shared__ int s_l[kDpThreads];
-            const int b = h.b;
-            const uint64_t P0r = W.P0[b], P2r = W.P2[b];
-            const int64_t P1r = W.P1[b];
-            float hi = INFINITY;
-            for (int l = kk + threadIdx.x; l <= b; l += blockDim.x) {
-                const Run q = run_of(W, l, P0r, P1r, P2r);
-                const float v = Ep[l] + u128_to_float_approx(fixed_num(q.s0, q.s1, q.s2, B, -1));
-                hi = fminf(hi, v * kMHi);
-            }
-            s_hi[threadIdx.x] = hi;
-            __syncthreads();
-            for (int o = blockDim.x / 2; o > 0; o >>= 1) {
-                if (threadIdx.x < o) s_hi[threadIdx.x] = fminf(s_hi[threadIdx.x], s_hi[threadIdx.x + o]);
-                __syncthreads();
-            }
-            const float best_hi = s_hi[0];
-            Best bst{INFINITY, 0};
-            for (int l = kk + threadIdx.x; l <= b; l += blockDim.x) {
-                const Run q = run_of(W, l, P0r, P1r, P2r);
-                const u128 num = fixed_num(q.s0, q.s1, q.s2, B, -1);
-                const float v = Ep[l] + u128_to_float_approx(num);
-                if (v * kMLo <= best_hi) take(bst, __dadd_rn(Dp[l - 1], u128_to_double_rn(num)), l);
-            }
-            s_v[threadIdx.x] = bst.v;
-            s_l[threadIdx.x] = bst.l;
-            __syncthreads();
-            for (int o = blockDim.x / 2; o > 0; o >>= 1) {
-                if (threadIdx.x < o) {
-                    Best a{s_v[threadIdx.x], s_l[threadIdx.x]};
-                    take(a, s_v[threadIdx.x + o], s_l[threadIdx.x + o]);
-                    s_v[threadIdx.x] = a.v;
-                    s_l[threadIdx.x] = a.l;
-                }
-                __syncthreads();
-            }
-            if (threadIdx.x == 0) {
-                Dk[b] = s_v[0];
-                Ak[b] = s_l[0];
-            }
-        }
-        if (r >= 0 && r <= B && r != h.b) {
-            Dk[r] = INFINITY;
-            Ak[r] = 0;
-        }
-        return;
-    }
-    if (g > B + 1) return;
+    const bool last = (kk == h.k_eff);
+    const bool active = kk <= h.k_eff && r <= h.b && (last ? (r == h.b) : (r >= kk));
     double d = INFINITY;
     int al = 0;
-    if (kk < h.k_eff && r >= kk && r <= h.b) {
-        // hint: the previous level's split at r, moved right by its share of
-        // the last cell
+    if (active) {
+        RowCtx c;
+        c.W = &W;
+        c.Dp = W.D + static_cast<size_t>(kk - 1) * n1;
+        c.Ep = W.E + static_cast<size_t>((kk - 1) & 1) * (n1 + 1);
+        c.P0r = W.P0[r];
+        c.P1r = W.P1[r];
+        c.P2r = W.P2[r];
+        c.B = B;
+        c.r = r;
+        c.last = last;
+        // hint: the previous level's split at r, moved by its share of the last cell
         const int hp = max(kk, W.A[static_cast<size_t>(kk - 1) * n1 + r]);
         const int hint = hp + (r - hp) / kk;
-        const Best bst = search_interior(W, Dp, Ep, kk, r, hint);
-        d = bst.v;
-        al = bst.l;
+        const Best b = search_row(c, kk, hint, lane, s_stack[warp]);
+        d = b.v;
+        al = b.l;
     }
-    if (r >= 0) {
-        Dk[r] = d;
-        Ak[r] = al;
+    if (lane == 0) {
+        W.D[static_cast<size_t>(kk) * n1 + r] = d;
+        W.A[static_cast<size_t>(kk) * n1 + r] = al;
+        const ff e = d_to_ff(d);
+        float2* En = W.E + static_cast<size_t>(kk & 1) * (n1 + 1);
+        En[r + 1] = make_float2(e.hi, e.lo);
+        if (r == 0) En[0] = make_float2(INFINITY, 0.0f);
     }
-    En[g] = __double2float_rn(d);
 }
 
 // Backtrack the splits into cell starts and levels (one thread).
@@ -461,9 +547,10 @@ extern "C" gefen_status_t gefen_refit_codebook(const float* x, int64_t n, const 
             return GEFEN_ECUDA;
     }
     k_dp_prefix<<<1, kPrefixThreads, 0, st>>>(h, bins, k, W);
-    const int grid = (bins + 2 + kDpThreads - 1) / kDpThreads;
-    k_dp_level1<<<grid, kDpThreads, 0, st>>>(bins, W);
-    for (int kk = 2; kk <= k; ++kk) k_dp_level<<<grid, kDpThreads, 0, st>>>(bins, kk, W);
+    const int grid1 = (bins + 2 + kDpThreads - 1) / kDpThreads;
+    k_dp_level1<<<grid1, kDpThreads, 0, st>>>(bins, W);
+    const int grid = (bins + 1 + kDpWarps - 1) / kDpWarps;
+    for (int kk = 2; kk <= k; ++kk) k_dp_level<<<grid, kDpWarps * 32, 0, st>>>(bins, kk, W);
     k_dp_backtrack<<<1, 32, 0, st>>>(bins, k, W, codebook_out, cell_start_out, cost_out);
     if (cudaGetLastError() != cudaSuccess) return GEFEN_ECUDA;
     return GEFEN_OK;

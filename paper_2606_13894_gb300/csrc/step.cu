@@ -44,7 +44,20 @@ struct Seg {
     int64_t unit_begin;  // first work unit (CTA) of this tensor in the launch
     int64_t per_unit;    // tile paths: blocks per tile; big path: chunks per block
     int64_t aux_begin;   // big path: first big-block index of this tensor
+    int64_t nblocks;     // numel / period
+    uint32_t pmagic;     // floor(2^32 / period) + 1: e / p == umulhi(e, pmagic) for e * p < 2^32
+    uint32_t pad;
 };
+
+inline void seg_fill(Seg& s, const gefen_tensor_t& x) {
+    s.elem_off = x.offset;
+    s.numel = x.numel;
+    s.period = x.period;
+    s.block_off = x.block_offset;
+    s.nblocks = x.numel / x.period;
+    s.pmagic = static_cast<uint32_t>((uint64_t(1) << 32) / static_cast<uint64_t>(x.period)) + 1u;
+    s.pad = 0;
+}
 
 struct HP {
     float beta1, omb1;  // beta1, 1 - beta1
@@ -203,7 +216,7 @@ __global__ void __launch_bounds__(kThreads) k_step_tile16(const __grid_constant_
     const HP& hp = L.hp;
     const int64_t p = S.period;
     const int64_t blk0 = (unit - S.unit_begin) * S.per_unit;
-    const int nblk = static_cast<int>(min(S.per_unit, S.numel / p - blk0));
+    const int nblk = static_cast<int>(min(S.per_unit, S.nblocks - blk0));
     const int64_t e0 = S.elem_off + blk0 * p;
     const int q = static_cast<int>(p >> 4);  // vectors per block
     const int nvec = nblk * q;
@@ -356,6 +369,367 @@ __global__ void __launch_bounds__(kThreads) k_step_tile16(const __grid_constant_
     }
 }
 
+// ------------------------------------------------ streamed tiles (bulk copy)
+// Persistent CTAs stream tiles of whole blocks (p % 16 == 0, p <= TILE)
+// through a STAGES-deep shared-memory ring: thread 0 issues cp.async.bulk
+// copies of theta, g and codes for tile i+STAGES-1 while every thread works on
+// tile i, and writes theta' and codes' back with bulk stores.  Decoding uses a
+// shared table; encoding maps x = m / s' to its cell of a uniform grid over
+// [-1, 1] whose record holds the number of midpoints below the cell and the next
+// three midpoints, so the nearest level is base + three compares (identical to
+// the binary search, which remains the fallback when a cell holds more than
+// three midpoints).
+constexpr int kLutCells = 512;
+constexpr float kLutGuard = 2.384185791015625e-07f;  // 2^-22, below every cell edge
+
+struct alignas(16) StreamTables {
+    float4 lut[kLutCells + 2];  // record c+1 for cell c in [-1, kLutCells]
+    float dec[kMaxLevels];
+    float mid[kMaxLevels + 4];
+};
+
+template <int TILE, int THREADS, int STAGES>
+struct alignas(128) StreamSmem {
+    unsigned char stage[STAGES][TILE * 7];  // theta f32 | g bf16 | codes u8
+    StreamTables tab;
+    float2 part[TILE / 8];   // per 8-element group (or per warp): (sum g^2, max |m|)
+    float2 blk[TILE / 16];   // per block: (step factor, 1/s')  [grad-only: (-, absmax)]
+    float sold[TILE / 16];   // per block: scale before the step
+    float vold[TILE / 16];   // per block: v before the step
+    unsigned long long bar[STAGES];
+};
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+// Waits for the barrier phase with the given parity; gives up after ~2^31
+// cycles (about a second) and returns false, so a lost copy cannot hang the GPU.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+    const long long t0 = clock64();
+    while (true) {
+        uint32_t ok;
+        asm volatile(
+            "{\n\t.reg .pred p;\n\t"
+            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+            "selp.u32 %0, 1, 0, p;\n\t}"
+            : "=r"(ok)
+            : "r"(bar), "r"(parity)
+            : "memory");
+        if (ok) return true;
+        if (clock64() - t0 > (1ll << 31)) return false;
+    }
+}
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+                 "l"(src), "r"(bytes), "r"(bar)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_s2g(void* dst, uint32_t src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst), "r"(src), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read_all() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+// Decode table, midpoints (padded with +inf) and the cell records.
+template <int THREADS>
+__device__ __forceinline__ int build_tables(const Ptrs& P, StreamTables& T, bool grad_only) {
+    const int t = threadIdx.x;
+    if (grad_only) return 0;
+    for (int i = t; i < kMaxLevels + 4; i += THREADS) {
+        if (i < kMaxLevels) T.dec[i] = i < P.k ? P.cb_dec[i] : 0.0f;
+        T.mid[i] = (i < P.k - 1) ? 0.5f * (P.cb_enc[i] + P.cb_enc[i + 1]) : INFINITY;
+    }
+    __syncthreads();
+    int bad = 0;
+    // cell(x) = floor(fma(x, G/2, G/2)) is within 2^-24 of exact in x: each
+    // record counts the midpoints below its cell minus a 2^-22 guard and holds
+    // the next three; its cell plus the guard on both sides may hold at most
+    // three midpoints, or the binary search is used instead.
+    for (int c = t - 1; c <= kLutCells; c += THREADS) {
+        const float lo = -1.0f + 2.0f * static_cast<float>(c) / kLutCells - kLutGuard;
+        const float hi = -1.0f + 2.0f * static_cast<float>(c + 1) / kLutCells + kLutGuard;
+        const int base = level_search(T.mid, lo);
+        const int upto = level_search(T.mid, hi);
+        bad |= (upto - base > 3);
+        T.lut[c + 1] = make_float4(__int_as_float(base), T.mid[base], T.mid[base + 1], T.mid[base + 2]);
+    }
+    return bad;
+}
+
+__device__ __forceinline__ int encode_lut(const StreamTables& T, bool lut_ok, float x) {
+    if (lut_ok) {
+        int c = __float2int_rd(__fmaf_rn(x, 0.5f * kLutCells, 0.5f * kLutCells));
+        c = min(max(c, -1), kLutCells);
+        const float4 r = T.lut[c + 1];
+        return __float_as_int(r.x) + (r.y < x) + (r.z < x) + (r.w < x);
+    }
+    return level_search(T.mid, x);
+}
+
+struct TileInfo {
+    int64_t e0;    // first element
+    int64_t bo;    // first block index into v / scale
+    int nelem;
+    int nblk;
+    int p;
+    uint32_t pmagic;  // floor(2^32 / p) + 1: e / p == umulhi(e, pmagic) for e, p < 2^16
+};
+
+__device__ __forceinline__ TileInfo tile_info(const Launch& L, int64_t unit) {
+    const Seg& S = L.seg[find_seg(L, unit)];
+    const int64_t p = S.period;
+    const int64_t blk0 = (unit - S.unit_begin) * S.per_unit;
+    TileInfo ti;
+    ti.nblk = static_cast<int>(min(S.per_unit, S.nblocks - blk0));
+    ti.p = static_cast<int>(p);
+    ti.nelem = ti.nblk * ti.p;
+    ti.e0 = S.elem_off + blk0 * p;
+    ti.bo = S.block_off + blk0;
+    ti.pmagic = S.pmagic;
+    return ti;
+}
+
+// A tile fits its stage iff it holds at most TILE elements, a multiple of 16
+// (so every copy is a whole number of 16-byte units).
+template <int TILE>
+__device__ __forceinline__ bool tile_fits(const TileInfo& ti) {
+    return ti.nelem > 0 && ti.nelem <= TILE && (ti.nelem & 15) == 0;
+}
+
+template <int TILE, int MODE>
+__device__ __forceinline__ void issue_tile(unsigned char* stage, uint32_t bar, const TileInfo& ti, const Ptrs& P) {
+    if (!tile_fits<TILE>(ti)) return;  // never copied; the consumer stops before waiting on it
+    const uint32_t n = static_cast<uint32_t>(ti.nelem);
+    if (MODE == kGradOnly) {
+        mbar_expect_tx(bar, 2u * n);
+        bulk_g2s(smem_u32(stage + 4 * TILE), P.grads + ti.e0, 2u * n, bar);
+    } else {
+        mbar_expect_tx(bar, 7u * n);
+        bulk_g2s(smem_u32(stage), P.params + ti.e0, 4u * n, bar);
+        bulk_g2s(smem_u32(stage + 4 * TILE), P.grads + ti.e0, 2u * n, bar);
+        bulk_g2s(smem_u32(stage + 6 * TILE), P.codes + ti.e0, n, bar);
+    }
+}
+
+template <int TILE, int THREADS, int STAGES, int MODE, int MINB>
+__global__ void __launch_bounds__(THREADS, MINB) k_step_stream(const __grid_constant__ Launch L, const Ptrs P, int* err) {
+    using Smem = StreamSmem<TILE, THREADS, STAGES>;
+    // each thread owns one group of 8 consecutive elements of the tile
+    static_assert(TILE == 8 * THREADS && THREADS >= TILE / 16 && THREADS % 32 == 0, "tile shape");
+    extern __shared__ __align__(128) unsigned char smem_raw[];
+    Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const HP& hp = L.hp;
+    const int64_t G = gridDim.x;
+
+    if (tid == 0) {
+        for (int s = 0; s < STAGES; ++s) mbar_init(smem_u32(&sm.bar[s]), 1u);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    const int bad = build_tables<THREADS>(P, sm.tab, MODE == kGradOnly);
+    const bool lut_ok = !__syncthreads_or(bad);
+    const int zero_code = (MODE != kGradOnly) ? level_search(sm.tab.mid, 0.0f) : 0;
+
+    if (tid == 0) {
+        for (int s = 0; s < STAGES - 1; ++s) {
+            const int64_t u = blockIdx.x + s * G;
+            if (u < L.nunits) issue_tile<TILE, MODE>(sm.stage[s], smem_u32(&sm.bar[s]), tile_info(L, u), P);
+        }
+    }
+    // block state of the first tile; later tiles' state is loaded one tile ahead
+    float r_sold = 0.0f, r_vold = 0.0f;
+    if (MODE != kGradOnly && blockIdx.x < L.nunits) {
+        const TileInfo t0 = tile_info(L, blockIdx.x);
+        if (tid < t0.nblk) { r_sold = P.scale[t0.bo + tid]; r_vold = P.v[t0.bo + tid]; }
+    }
+
+    for (int it = 0;; ++it) {
+        const int64_t u = blockIdx.x + static_cast<int64_t>(it) * G;
+        if (u >= L.nunits) break;
+        const int s = it % STAGES;
+        const uint32_t parity = static_cast<uint32_t>((it / STAGES) & 1);
+        const TileInfo ti = tile_info(L, u);
+        if (!tile_fits<TILE>(ti)) {
+            // a tile the host planned too large: nothing was copied for it.
+            // Wait (bounded) for the copies already issued for later tiles,
+            // flag the error and stop.
+            for (int j = 1; j < STAGES; ++j) {
+                const int64_t uj = u + static_cast<int64_t>(j) * G;
+                if (uj >= L.nunits || !tile_fits<TILE>(tile_info(L, uj))) continue;
+                mbar_wait(smem_u32(&sm.bar[(it + j) % STAGES]), static_cast<uint32_t>(((it + j) / STAGES) & 1));
+            }
+            if (tid == 0) atomicExch(err, 2);
+            break;
+        }
+        if (MODE != kGradOnly) {
+            if (tid < ti.nblk) { sm.sold[tid] = r_sold; sm.vold[tid] = r_vold; }
+            if (u + G < L.nunits) {
+                const TileInfo tn = tile_info(L, u + G);
+                if (tid < tn.nblk) { r_sold = P.scale[tn.bo + tid]; r_vold = P.v[tn.bo + tid]; }
+            }
+        }
+        const bool ok = mbar_wait(smem_u32(&sm.bar[s]), parity);
+        if (__syncthreads_or(!ok)) {
+            if (tid == 0) atomicExch(err, 1);
+            break;
+        }
+        unsigned char* st = sm.stage[s];
+        float* sth = reinterpret_cast<float*>(st);
+        const uint16_t* sg = reinterpret_cast<const uint16_t*>(st + 4 * TILE);
+        uint8_t* sc = st + 6 * TILE;
+        const int q = ti.p >> 3;  // 8-element groups per block (p % 16 == 0)
+        const float pf = static_cast<float>(ti.p);
+        // a block whose groups all sit in one warp finishes in phase 1
+        const bool seg = (q <= 32) && ((32 % q) == 0);
+        const bool warp_part = !seg && (q % 32 == 0);
+        auto finish = [&](int b, float g2, float mx) {
+            if (MODE == kGradOnly) {
+                sm.blk[b] = make_float2(0.0f, mx);
+            } else {
+                const float vn = fmaf(hp.beta2, sm.vold[b], hp.omb2 * (g2 / pf));
+                P.v[ti.bo + b] = vn;
+                P.scale[ti.bo + b] = mx;
+                const float fac = hp.lr_bc1 / (sqrtf(vn * hp.inv_bc2) + hp.eps);
+                sm.blk[b] = make_float2(fac, mx > 0.0f ? 1.0f / mx : 0.0f);
+            }
+        };
+
+        // phase 1: decode m, partials over the thread's 8 elements
+        const int e = tid * 8;
+        const bool live = e < ti.nelem;
+        const int b = static_cast<int>(__umulhi(static_cast<uint32_t>(e), ti.pmagic));
+        float m[8];
+        float g2 = 0.0f, mx = 0.0f;
+        if (live) {
+            const uint4 gw = *reinterpret_cast<const uint4*>(sg + e);
+            const uint32_t gws[4] = {gw.x, gw.y, gw.z, gw.w};
+            if (MODE == kGradOnly) {
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    m[2 * j] = bf16_lo(gws[j]);
+                    m[2 * j + 1] = bf16_hi(gws[j]);
+                }
+#pragma unroll
+                for (int j = 0; j < 8; ++j) mx = fmaxf(mx, fabsf(m[j]));
+            } else {
+                const uint2 cw = *reinterpret_cast<const uint2*>(sc + e);
+                const float b1s = hp.beta1 * sm.sold[b];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    const float g = (j & 1) ? bf16_hi(gws[j >> 1]) : bf16_lo(gws[j >> 1]);
+                    const uint32_t c = ((j < 4 ? cw.x : cw.y) >> (8 * (j & 3))) & 0xFFu;
+                    const float mm = fmaf(hp.omb1, g, b1s * sm.tab.dec[c]);
+                    m[j] = mm;
+                    g2 = fmaf(g, g, g2);
+                    mx = fmaxf(mx, fabsf(mm));
+                }
+            }
+        }
+        if (seg) {
+            for (int o = q >> 1; o > 0; o >>= 1) {
+                g2 += __shfl_xor_sync(0xffffffffu, g2, o);
+                mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+            }
+            if (live && (tid % q) == 0) finish(b, g2, mx);
+        } else if (warp_part) {
+            g2 = warp_sum(g2);
+            mx = warp_max(mx);
+            if (lane == 0) sm.part[tid >> 5] = make_float2(g2, mx);
+        } else {
+            sm.part[tid] = make_float2(g2, mx);
+        }
+        __syncthreads();
+        if (!seg) {
+            // remaining block reductions over the stored partials (fixed order)
+            const int per = warp_part ? (q >> 5) : q;
+            for (int bb = warp; bb < ti.nblk; bb += THREADS / 32) {
+                float s2 = 0.0f, sx = 0.0f;
+                for (int t = lane; t < per; t += 32) {
+                    const float2 pp = sm.part[bb * per + t];
+                    s2 += pp.x;
+                    sx = fmaxf(sx, pp.y);
+                }
+                s2 = warp_sum(s2);
+                sx = warp_max(sx);
+                if (lane == 0) finish(bb, s2, sx);
+            }
+            __syncthreads();
+        }
+
+        // phase 2: update and re-encode into the stage, x to the staging buffer
+        if (live) {
+            const float2 bs = sm.blk[b];
+            float x[8];
+            if (MODE == kGradOnly) {
+#pragma unroll
+                for (int j = 0; j < 8; ++j) x[j] = bs.y > 0.0f ? __fdiv_rn(m[j], bs.y) : __int_as_float(0x7fffffff);
+            } else {
+                float4* tp = reinterpret_cast<float4*>(sth + e);
+                float4 t0 = tp[0], t1 = tp[1];
+                t0.x = fmaf(-bs.x, m[0], hp.decay * t0.x);
+                t0.y = fmaf(-bs.x, m[1], hp.decay * t0.y);
+                t0.z = fmaf(-bs.x, m[2], hp.decay * t0.z);
+                t0.w = fmaf(-bs.x, m[3], hp.decay * t0.w);
+                t1.x = fmaf(-bs.x, m[4], hp.decay * t1.x);
+                t1.y = fmaf(-bs.x, m[5], hp.decay * t1.y);
+                t1.z = fmaf(-bs.x, m[6], hp.decay * t1.z);
+                t1.w = fmaf(-bs.x, m[7], hp.decay * t1.w);
+                tp[0] = t0;
+                tp[1] = t1;
+                uint32_t w0 = 0, w1 = 0;
+                if (bs.y > 0.0f) {
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        x[j] = m[j] * bs.y;
+                        const uint32_t c = static_cast<uint32_t>(encode_lut(sm.tab, lut_ok, x[j]));
+                        if (j < 4) w0 |= c << (8 * j); else w1 |= c << (8 * (j - 4));
+                    }
+                } else {
+                    const uint32_t z = static_cast<uint32_t>(zero_code) * 0x01010101u;
+                    w0 = w1 = z;
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) x[j] = __int_as_float(0x7fffffff);
+                }
+                *reinterpret_cast<uint2*>(sc + e) = make_uint2(w0, w1);
+            }
+            if (MODE != kPlain) {
+                float4* xs = reinterpret_cast<float4*>(P.xstage + ti.e0 + e);
+                __stcs(xs, make_float4(x[0], x[1], x[2], x[3]));
+                __stcs(xs + 1, make_float4(x[4], x[5], x[6], x[7]));
+            }
+        }
+        if (MODE != kGradOnly) fence_proxy_async();
+        __syncthreads();
+        if (tid == 0) {
+            if (MODE != kGradOnly) {
+                const uint32_t n = static_cast<uint32_t>(ti.nelem);
+                bulk_s2g(P.params + ti.e0, smem_u32(sth), 4u * n);
+                bulk_s2g(P.codes + ti.e0, smem_u32(sc), n);
+            }
+            bulk_commit();
+            // Refill the stage tile it-1 used with tile it+STAGES-1.  Its store
+            // was committed an iteration ago: wait until only this tile's
+            // store may still be reading shared memory.
+            const int64_t un = u + static_cast<int64_t>(STAGES - 1) * G;
+            if (un < L.nunits) {
+                asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+                const int sn = (it + STAGES - 1) % STAGES;
+                issue_tile<TILE, MODE>(sm.stage[sn], smem_u32(&sm.bar[sn]), tile_info(L, un), P);
+            }
+        }
+    }
+    if (tid == 0) bulk_wait_all();
+}
+
 // ------------------------------------------- generic p <= 2048 (scalar)
 // Any period: a tile of whole blocks (<= kGenericTile elements), element
 // partials in shared memory, per-block reductions, then the update.
@@ -371,7 +745,7 @@ __global__ void __launch_bounds__(kThreads) k_step_generic(const __grid_constant
     const HP& hp = L.hp;
     const int64_t p = S.period;
     const int64_t blk0 = (unit - S.unit_begin) * S.per_unit;
-    const int nblk = static_cast<int>(min(S.per_unit, S.numel / p - blk0));
+    const int nblk = static_cast<int>(min(S.per_unit, S.nblocks - blk0));
     const int ne = nblk * static_cast<int>(p);
     const int64_t e0 = S.elem_off + blk0 * p;
     const int64_t bo = S.block_off + blk0;
@@ -667,25 +1041,36 @@ __global__ void __launch_bounds__(kThreads) k_big_apply(const __grid_constant__ 
 }
 
 // ------------------------------------------------------------- host side
-enum PathClass { kP1 = 0, kT16V2, kT16V4, kGeneric, kBigAligned, kBigUnaligned, kNumClasses };
+enum PathClass { kP1 = 0, kS4K, kS8K, kT16V4, kGeneric, kBigAligned, kBigUnaligned, kNumClasses };
+
+// p <= 4096: two 512-thread CTAs per SM, 3-stage rings of 28 KB tiles;
+// p <= 8192: one 1024-thread CTA per SM, 3-stage ring of 56 KB tiles
+constexpr int kS4KTile = 4096, kS4KThreads = 512, kS4KStages = 3, kS4KMinBlocks = 2;
+constexpr int kS8KTile = 8192, kS8KThreads = 1024, kS8KStages = 3, kS8KMinBlocks = 1;
 
 PathClass classify(int64_t p) {
     if (p == 1) return kP1;
-    if (p % 16 == 0 && p <= kThreads * 2 * 16) return kT16V2;
+    if (p % 16 == 0 && p <= kS4KTile) return kS4K;
+    if (p % 16 == 0 && p <= kS8KTile) return kS8K;
     if (p % 16 == 0 && p <= kTile16Max) return kT16V4;
     if (p <= kGenericTile) return kGeneric;
     return (p % 16 == 0) ? kBigAligned : kBigUnaligned;
 }
 
-int64_t units_of(PathClass c, const gefen_tensor_t& t, int64_t* per_unit) {
+int64_t units_of(PathClass c, const gefen_tensor_t& t, int64_t* per_unit, int64_t tile_cap = 0) {
     const int64_t p = t.period, nb = t.numel / p;
+    if (tile_cap > 0) {  // streamed classes: whole blocks per tile of the kernel's own size
+        *per_unit = std::max<int64_t>(1, tile_cap / p);
+        return (nb + *per_unit - 1) / *per_unit;
+    }
     switch (c) {
         case kP1:
             *per_unit = 1;
             return (t.numel + 4 * kThreads - 1) / (4 * kThreads);
-        case kT16V2:
+        case kS4K:
+        case kS8K:
         case kT16V4: {
-            const int64_t cap = (c == kT16V2) ? kThreads * 2 * 16 : kThreads * 4 * 16;
+            const int64_t cap = (c == kS4K) ? kS4KTile : (c == kS8K) ? kS8KTile : kThreads * 4 * 16;
             *per_unit = std::max<int64_t>(1, cap / p);
             return (nb + *per_unit - 1) / *per_unit;
         }
@@ -721,12 +1106,16 @@ Plan make_plan(const gefen_tensor_t* t, int32_t n) {
 }
 
 struct WsLayout {
-    size_t part_g2, part_mx, blk_state, xstage, total;
+    size_t header, part_g2, part_mx, blk_state, xstage, total;
 };
 
+// Workspace: a 256-byte header (word 0: set when a bounded device wait gave
+// up), then big-block partials and block state, then the histogram staging.
 WsLayout ws_layout(const Plan& pl, uint32_t flags) {
     WsLayout w;
     size_t o = 0;
+    w.header = o;
+    o += kWsAlign;
     w.part_g2 = o;
     o += align_up(static_cast<size_t>(pl.big_chunks) * sizeof(double));
     w.part_mx = o;
@@ -763,7 +1152,7 @@ bool validate_tensors(const gefen_tensor_t* t, int32_t n) {
 // per group through `kernel(L, units)`.
 template <typename K>
 cudaError_t launch_class(K kernel, Launch& L, const std::vector<int>& ids, const gefen_tensor_t* t,
-                         PathClass c) {
+                         PathClass c, int64_t tile_cap = 0) {
     size_t i = 0;
     while (i < ids.size()) {
         L.nseg = 0;
@@ -771,13 +1160,11 @@ cudaError_t launch_class(K kernel, Launch& L, const std::vector<int>& ids, const
         for (; i < ids.size() && L.nseg < kMaxSegs; ++i) {
             const gefen_tensor_t& x = t[ids[i]];
             Seg& s = L.seg[L.nseg++];
-            s.elem_off = x.offset;
-            s.numel = x.numel;
-            s.period = x.period;
-            s.block_off = x.block_offset;
+            seg_fill(s, x);
             s.unit_begin = units;
             s.aux_begin = 0;
-            units += units_of(c, x, &s.per_unit);
+            if (tile_cap > 0 && x.period > tile_cap) return cudaErrorInvalidValue;  // planning error
+            units += units_of(c, x, &s.per_unit, tile_cap);
         }
         L.nunits = units;
         if (units == 0) continue;
@@ -788,14 +1175,35 @@ cudaError_t launch_class(K kernel, Launch& L, const std::vector<int>& ids, const
     return cudaSuccess;
 }
 
+template <int TILE, int THREADS, int STAGES, int MINB, int MODE>
+cudaError_t launch_stream(Launch& L, const std::vector<int>& ids, const gefen_tensor_t* t, PathClass c,
+                          const Ptrs& P, int* err, cudaStream_t st) {
+    auto kern = k_step_stream<TILE, THREADS, STAGES, MODE, MINB>;
+    const int smem = static_cast<int>(sizeof(StreamSmem<TILE, THREADS, STAGES>));
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
+    if (e != cudaSuccess) return e;
+    int per_sm = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, THREADS, smem);
+    if (e != cudaSuccess) return e;
+    const int64_t cap = static_cast<int64_t>(std::max(1, per_sm)) * device_sm_count();
+    return launch_class(
+        [&](Launch& LL, int64_t u) {
+            kern<<<dim3(static_cast<unsigned>(std::min(u, cap))), THREADS, smem, st>>>(LL, P, err);
+        },
+        L, ids, t, c, TILE);
+}
+
 template <int MODE>
-cudaError_t run_step(const Plan& pl, const gefen_tensor_t* t, Launch& L, const Ptrs& P, cudaStream_t st) {
+cudaError_t run_step(const Plan& pl, const gefen_tensor_t* t, Launch& L, const Ptrs& P, int* err, cudaStream_t st) {
     cudaError_t e;
     e = launch_class([&](Launch& LL, int64_t u) { k_step_p1<MODE><<<dim3(u), kThreads, 0, st>>>(LL, P); },
                      L, pl.idx[kP1], t, kP1);
     if (e != cudaSuccess) return e;
-    e = launch_class([&](Launch& LL, int64_t u) { k_step_tile16<2, MODE><<<dim3(u), kThreads, 0, st>>>(LL, P); },
-                     L, pl.idx[kT16V2], t, kT16V2);
+    e = launch_stream<kS4KTile, kS4KThreads, kS4KStages, kS4KMinBlocks, MODE>(L, pl.idx[kS4K], t, kS4K, P, err, st);
+    if (e != cudaSuccess) return e;
+    e = launch_stream<kS8KTile, kS8KThreads, kS8KStages, kS8KMinBlocks, MODE>(L, pl.idx[kS8K], t, kS8K, P, err, st);
     if (e != cudaSuccess) return e;
     e = launch_class([&](Launch& LL, int64_t u) { k_step_tile16<4, MODE><<<dim3(u), kThreads, 0, st>>>(LL, P); },
                      L, pl.idx[kT16V4], t, kT16V4);
@@ -815,10 +1223,7 @@ cudaError_t run_step(const Plan& pl, const gefen_tensor_t* t, Launch& L, const P
             for (; i < ids.size() && L.nseg < kMaxSegs; ++i) {
                 const gefen_tensor_t& x = t[ids[i]];
                 Seg& s = L.seg[L.nseg++];
-                s.elem_off = x.offset;
-                s.numel = x.numel;
-                s.period = x.period;
-                s.block_off = x.block_offset;
+                seg_fill(s, x);
                 s.unit_begin = units;
                 s.aux_begin = blocks;
                 units += units_of(static_cast<PathClass>(cls), x, &s.per_unit);
@@ -871,7 +1276,7 @@ extern "C" gefen_status_t gefen_step(const gefen_tensor_t* tensors, int32_t nten
     if (want_hist && (hist == nullptr || hist_bins < 1 || hist_bins > GEFEN_MAX_BINS)) return GEFEN_EINVAL;
     const Plan pl = make_plan(tensors, ntensors);
     const WsLayout wl = ws_layout(pl, flags);
-    if (workspace_bytes < wl.total || (wl.total > 0 && workspace == nullptr)) return GEFEN_ENOMEM;
+    if (workspace_bytes < wl.total || workspace == nullptr) return GEFEN_ENOMEM;
     if (reinterpret_cast<uintptr_t>(workspace) % kWsAlign) return GEFEN_EINVAL;
     if (gefen_status_t s = check_device(); s != GEFEN_OK) return s;
 
@@ -906,9 +1311,10 @@ extern "C" gefen_status_t gefen_step(const gefen_tensor_t* tensors, int32_t nten
     }
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     cudaError_t e;
-    if (grad_only) e = run_step<kGradOnly>(pl, tensors, L, P, st);
-    else if (flags & GEFEN_HIST) e = run_step<kHist>(pl, tensors, L, P, st);
-    else e = run_step<kPlain>(pl, tensors, L, P, st);
+    int* err = reinterpret_cast<int*>(ws + wl.header);
+    if (grad_only) e = run_step<kGradOnly>(pl, tensors, L, P, err, st);
+    else if (flags & GEFEN_HIST) e = run_step<kHist>(pl, tensors, L, P, err, st);
+    else e = run_step<kPlain>(pl, tensors, L, P, err, st);
     if (e != cudaSuccess) return GEFEN_ECUDA;
     if (want_hist) {
         std::vector<HistRange> rr;
@@ -919,4 +1325,15 @@ extern "C" gefen_status_t gefen_step(const gefen_tensor_t* tensors, int32_t nten
             return GEFEN_ECUDA;
     }
     return GEFEN_OK;
+}
+
+extern "C" gefen_status_t gefen_step_status(void* workspace, gefen_stream_t stream) {
+    if (workspace == nullptr || reinterpret_cast<uintptr_t>(workspace) % kWsAlign) return GEFEN_EINVAL;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    int word = 0;
+    if (cudaMemcpyAsync(&word, workspace, sizeof(word), cudaMemcpyDeviceToHost, st) != cudaSuccess) return GEFEN_ECUDA;
+    if (cudaStreamSynchronize(st) != cudaSuccess) return GEFEN_ECUDA;
+    if (word == 0) return GEFEN_OK;
+    if (cudaMemsetAsync(workspace, 0, sizeof(word), st) != cudaSuccess) return GEFEN_ECUDA;
+    return GEFEN_ETIMEOUT;
 }

@@ -43,6 +43,7 @@ class gefen_hparams_t(ctypes.Structure):
 
 
 EXPORTS = ("gefen_status_string", "gefen_sync_status", "gefen_step_workspace_size", "gefen_step",
+           "gefen_step_status",
            "gefen_refit_workspace_size", "gefen_refit_codebook", "gefen_refit_status",
            "gefen_refit_tables", "gefen_infer_workspace_size", "gefen_infer_blocks")
 
@@ -74,6 +75,8 @@ def load(build_if_needed: bool = True):
         L.gefen_step_workspace_size.restype = sz
         L.gefen_step.argtypes = [P, i32, P, P, P, P, P, P, P, i32, gefen_hparams_t, P, i32, P, sz, P]
         L.gefen_step.restype = ctypes.c_int
+        L.gefen_step_status.argtypes = [P, P]
+        L.gefen_step_status.restype = ctypes.c_int
         L.gefen_refit_workspace_size.argtypes = [i32, i32]
         L.gefen_refit_workspace_size.restype = sz
         L.gefen_refit_codebook.argtypes = [P, i64, P, i32, i32, P, P, P, P, P, sz, P]
@@ -118,10 +121,11 @@ def tensor_table(entries: Iterable[Sequence[int]]):
 
 
 def workspace(nbytes: int, device=None) -> torch.Tensor:
-    """A device buffer of at least nbytes, 256-byte aligned (torch allocation)."""
+    """A zero-filled device buffer of at least nbytes, 256-byte aligned (torch
+    allocation)."""
     if device is None:
         device = torch.device("cuda", torch.cuda.current_device())
-    buf = torch.empty(max(1, int(nbytes)) + WS_ALIGN, dtype=torch.uint8, device=device)
+    buf = torch.zeros(max(1, int(nbytes)) + WS_ALIGN, dtype=torch.uint8, device=device)
     off = (-buf.data_ptr()) % WS_ALIGN
     return buf[off:off + max(1, int(nbytes))]
 
@@ -158,6 +162,12 @@ def gefen_step(table, params, grads, codes, v, scale, codebook_dec, codebook_enc
                            _ptr(workspace_buf), workspace_buf.numel(), _stream(stream))
     _check("gefen_step", st)
     return workspace_buf
+
+
+def gefen_step_status(workspace_buf, stream=None):
+    """Raises GefenError(GEFEN_ETIMEOUT) if a step using this workspace gave up
+    a bounded wait (its outputs are then invalid); waits for the stream."""
+    _check("gefen_step_status", load().gefen_step_status(_ptr(workspace_buf), _stream(stream)))
 
 
 def gefen_refit_workspace_size(bins: int, k: int) -> int:

@@ -39,8 +39,9 @@ def _table(entries):
 
 
 def test_step_workspace_sizes_follow_the_plan():
-    # small blocks need no scratch; big blocks need per-chunk partials
-    assert G.gefen_step_workspace_size(_table([(0, 4096, 64, 0)])) == 0
+    # small blocks need only the 256-byte status header; big blocks need
+    # per-chunk partials as well
+    assert G.gefen_step_workspace_size(_table([(0, 4096, 64, 0)])) == 256
     big = G.gefen_step_workspace_size(_table([(0, 1 << 20, 1 << 20, 0)]))
     assert big > 0
     hist = G.gefen_step_workspace_size(_table([(0, 4096, 64, 0)]), G.GEFEN_HIST)
@@ -102,6 +103,8 @@ def test_step_rejects_bad_scalars_and_pointers():
     assert _step(t, hp=_hp(flags=G.GEFEN_HIST), hist=FAKE, bins=70000) == G.GEFEN_EINVAL
     big = _table([(0, 1 << 20, 1 << 20, 0)])
     assert _step(big) == G.GEFEN_ENOMEM  # scratch needed but none given
+    assert _step(t) == G.GEFEN_ENOMEM    # the status header is always needed
+    assert _step(t, ws=ctypes.c_void_p((1 << 20) + 64), ws_bytes=4096) == G.GEFEN_EINVAL  # misaligned
 
 
 def test_refit_and_infer_reject_bad_arguments():

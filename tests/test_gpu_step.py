@@ -13,13 +13,16 @@ pytestmark = pytest.mark.gpu
 
 PATH_CASES = {
     "p1": [(1000, 1), (4096, 1)],
-    "tile16_v2": [(64 * 300, 64), (2048 * 7, 2048), (8192 * 3, 8192), (16 * 999, 16), (768 * 5, 768)],
+    "stream4k": [(64 * 300, 64), (2048 * 7, 2048), (4096 * 3, 4096), (16 * 999, 16), (768 * 5, 768), (48 * 401, 48)],
+    "stream8k": [(8192 * 3, 8192), (6144 * 5, 6144), (4112 * 4, 4112)],
     "tile16_v4": [(16384 * 3, 16384), (12288 * 2, 12288)],
     "generic": [(3 * 1000, 3), (7 * 333, 7), (100 * 50, 100), (2047 * 3, 2047), (2 * 4001, 2)],
     "big_aligned": [(65536 * 2, 65536), (20000 * 3, 20000), (1 << 20, 1 << 20)],
     "big_unaligned": [(30001 * 2, 30001), (8193 * 3, 8193)],
-    "mixed": [(1000, 1), (64 * 40, 64), (3 * 77, 3), (40000, 40000), (16384, 16384), (0, 4)],
+    "mixed": [(1000, 1), (64 * 40, 64), (3 * 77, 3), (40000, 40000), (16384, 16384), (0, 4), (8192, 8192)],
 }
+# several tiles per persistent CTA, so the shared-memory stage ring wraps
+RING_CASES = [(64 * 100_000, 64), (8192 * 1500, 8192), (2048 * 4000, 2048)]
 
 
 def _run(cases, steps=3, k=256, hist_mode=0, bins=4096, seed=0, switch=False, zero_blocks=0.0, hp=None):
@@ -42,7 +45,7 @@ def _run(cases, steps=3, k=256, hist_mode=0, bins=4096, seed=0, switch=False, ze
         hist = torch.zeros(bins, dtype=torch.int64, device="cuda") if hist_mode else None
         ws = G.gefen_step(A.table, A.theta, gb, A.codes, A.v, A.s, d_cb, enc, step=t, flags=flags,
                           hist=hist, workspace_buf=ws, **hp)
-        G.gefen_sync_status()
+        G.gefen_step_status(ws)
         th, cd, v, s, h = U.oracle_step(A, pre, gbits, cb, cbe, t, hp, hist_mode=hist_mode, bins=bins)
         got = A.host()
         if hist_mode == 2:
@@ -87,12 +90,12 @@ def test_step_parity_per_path(path):
     _run(PATH_CASES[path], steps=3)
 
 
-@pytest.mark.parametrize("path", ["tile16_v2", "generic", "big_aligned", "big_unaligned", "p1"])
+@pytest.mark.parametrize("path", ["stream4k", "stream8k", "generic", "big_aligned", "big_unaligned", "p1"])
 def test_step_histogram_of_normalised_momentum(path):
     _run(PATH_CASES[path], steps=2, hist_mode=1, bins=4096)
 
 
-@pytest.mark.parametrize("path", ["tile16_v2", "mixed", "big_unaligned"])
+@pytest.mark.parametrize("path", ["stream4k", "mixed", "big_unaligned"])
 def test_step_histogram_65536_cells(path):
     _run(PATH_CASES[path], steps=2, hist_mode=1, bins=65536)
 
@@ -112,7 +115,7 @@ def test_zero_blocks_and_16_level_codebook():
 
 
 def test_hyperparameter_variants():
-    _run(PATH_CASES["tile16_v2"], steps=2, hp=dict(beta1=0.0, beta2=0.95, weight_decay=0.1, lr=6e-4))
+    _run(PATH_CASES["stream4k"], steps=2, hp=dict(beta1=0.0, beta2=0.95, weight_decay=0.1, lr=6e-4))
     _run(PATH_CASES["generic"], steps=2, hp=dict(beta1=0.5, beta2=0.0, weight_decay=0.0, lr=1e-2))
 
 
@@ -128,3 +131,14 @@ def test_step_leaves_untouched_padding_alone():
     G.gefen_step(A.table, A.theta, gb, A.codes, A.v, A.s, d, d, step=1, **U.HP)
     torch.cuda.synchronize()
     assert torch.all(A.theta[100:128] == 7.0) and torch.all(A.codes[100:128] == 9)
+
+
+def test_stream_ring_wraps_over_many_tiles():
+    """Large enough that every persistent CTA streams many tiles through its
+    three shared-memory stages (16-level codebook keeps the oracle quick)."""
+    _run(RING_CASES, steps=2, k=16)
+
+
+def test_stream_ring_histogram_and_grad_only():
+    _run(RING_CASES[:1], steps=1, k=16, hist_mode=1, bins=4096)
+    _run(RING_CASES, steps=1, k=16, hist_mode=2, bins=65536)
