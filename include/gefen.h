@@ -186,6 +186,33 @@ gefen_status_t gefen_refit_tables(const void* workspace, int32_t bins, int32_t k
                                   gefen_stream_t stream);
 
 /* -------------------------------------------------------------------------
+ * gefen_refit_codebook_static -- gefen_refit_codebook without a workspace.
+ * The paper has no counterpart: this entry point exists for callers that
+ * cannot allocate device memory when they refit -- a host program whose
+ * memory is reserved up front by a framework's caching allocator or a serving
+ * runtime (so no workspace can be carved out), or a caller that must not
+ * synchronise the device, which cudaFree (and at times cudaMalloc) do.
+ *
+ * Same inputs, outputs and results as gefen_refit_codebook(); the scratch is
+ * one device array inside the library, sized for bins <= 4096 and k <= 256
+ * (about 12.9 MB, held on every device that loads the library until the
+ * process exits).  Larger requests return GEFEN_EUNSUPPORTED.  It allocates
+ * nothing: no cudaMalloc, cudaFree or allocating library call.
+ *
+ * The first call on a device looks up the array's device address for that
+ * device (once), so make it before any stream capture on that device.  All
+ * calls share the one array and it keeps the last call's contents (the refit
+ * clears what it needs); calls whose work overlaps on the GPU -- different
+ * streams, or different host threads -- race on it and must be ordered by the
+ * caller.  The device-side overflow check of the moments is not reported by
+ * this entry point; gefen_refit_codebook() with gefen_refit_status() reports it.
+ * ------------------------------------------------------------------------- */
+gefen_status_t gefen_refit_codebook_static(const float* x, int64_t n, const uint64_t* hist_in,
+                                           int32_t bins, int32_t k, float* codebook_out,
+                                           uint64_t* hist_out, int32_t* cell_start_out,
+                                           double* cost_out, gefen_stream_t stream);
+
+/* -------------------------------------------------------------------------
  * gefen_infer_blocks -- Algorithm 2 (Automatic Block Partitioning) for one
  * flattened gradient tensor g (bf16 bits, device, numel elements).
  *

@@ -25,6 +25,7 @@
 // scan bit for bit.
 #include <algorithm>
 #include <cmath>
+#include <mutex>
 
 #include "common.cuh"
 #include "internal.h"
@@ -581,4 +582,57 @@ extern "C" gefen_status_t gefen_refit_tables(const void* workspace, int32_t bins
         cudaMemcpyAsync(argl_out, ws + L.A, cnt * sizeof(int32_t), cudaMemcpyDeviceToDevice, st) != cudaSuccess)
         return GEFEN_ECUDA;
     return GEFEN_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Refit without a caller workspace.  The scratch the refit needs lives in one
+// file-scope device array sized for the largest request it accepts: 4096
+// histogram cells (16 cells per level at 256 levels) and 256 levels.  Every
+// device that loads this library holds the array until the process exits.
+namespace {
+
+constexpr int kStaticMaxBins = 4096;
+constexpr int kStaticMaxLevels = 256;
+
+constexpr size_t cx_align(size_t x) { return (x + kWsAlign - 1) / kWsAlign * kWsAlign; }
+// Mirrors dp_layout(kStaticMaxBins, kStaticMaxLevels).
+constexpr size_t kStaticScratchBytes =
+    cx_align(sizeof(Header)) + cx_align(size_t(kStaticMaxBins) * sizeof(uint64_t)) +
+    cx_align(size_t(kStaticMaxBins + 1) * sizeof(int32_t)) + 3 * cx_align(size_t(kStaticMaxBins + 1) * 8) +
+    cx_align(size_t(kStaticMaxLevels + 1) * (kStaticMaxBins + 1) * sizeof(double)) +
+    cx_align(size_t(kStaticMaxLevels + 1) * (kStaticMaxBins + 1) * sizeof(int32_t)) +
+    cx_align(2 * size_t(kStaticMaxBins + 2) * sizeof(float2));
+
+__device__ __align__(256) unsigned char g_refit_scratch[kStaticScratchBytes];
+
+// Device address of the array, looked up once per device.
+std::mutex g_scratch_mu;
+void* g_scratch_addr[64] = {nullptr};
+
+gefen_status_t static_scratch(void** out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return GEFEN_ECUDA;
+    std::lock_guard<std::mutex> g(g_scratch_mu);
+    if (g_scratch_addr[dev] == nullptr) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_refit_scratch) != cudaSuccess || p == nullptr) return GEFEN_ECUDA;
+        g_scratch_addr[dev] = p;
+    }
+    *out = g_scratch_addr[dev];
+    return GEFEN_OK;
+}
+
+}  // namespace
+
+extern "C" gefen_status_t gefen_refit_codebook_static(const float* x, int64_t n, const uint64_t* hist_in,
+                                                      int32_t bins, int32_t k, float* codebook_out,
+                                                      uint64_t* hist_out, int32_t* cell_start_out,
+                                                      double* cost_out, gefen_stream_t stream) {
+    if (bins < 1 || k < 2 || codebook_out == nullptr || (x == nullptr && hist_in == nullptr)) return GEFEN_EINVAL;
+    if (bins > kStaticMaxBins || k > kStaticMaxLevels) return GEFEN_EUNSUPPORTED;
+    if (dp_layout(bins, k).total > kStaticScratchBytes) return GEFEN_EUNSUPPORTED;
+    void* scratch = nullptr;
+    if (gefen_status_t s = static_scratch(&scratch); s != GEFEN_OK) return s;
+    return gefen_refit_codebook(x, n, hist_in, bins, k, codebook_out, hist_out, cell_start_out, cost_out, scratch,
+                                kStaticScratchBytes, stream);
 }

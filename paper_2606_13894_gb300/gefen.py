@@ -45,7 +45,8 @@ class gefen_hparams_t(ctypes.Structure):
 EXPORTS = ("gefen_status_string", "gefen_sync_status", "gefen_step_workspace_size", "gefen_step",
            "gefen_step_status",
            "gefen_refit_workspace_size", "gefen_refit_codebook", "gefen_refit_status",
-           "gefen_refit_tables", "gefen_infer_workspace_size", "gefen_infer_blocks")
+           "gefen_refit_tables", "gefen_infer_workspace_size", "gefen_infer_blocks",
+           "gefen_refit_codebook_static")
 
 _lib = None
 _lock = threading.Lock()
@@ -81,6 +82,8 @@ def load(build_if_needed: bool = True):
         L.gefen_refit_workspace_size.restype = sz
         L.gefen_refit_codebook.argtypes = [P, i64, P, i32, i32, P, P, P, P, P, sz, P]
         L.gefen_refit_codebook.restype = ctypes.c_int
+        L.gefen_refit_codebook_static.argtypes = [P, i64, P, i32, i32, P, P, P, P, P]
+        L.gefen_refit_codebook_static.restype = ctypes.c_int
         L.gefen_refit_status.argtypes = [P, ctypes.POINTER(i32), P]
         L.gefen_refit_status.restype = ctypes.c_int
         L.gefen_refit_tables.argtypes = [P, i32, i32, P, P, P]
@@ -191,6 +194,27 @@ def gefen_refit_codebook(*, bins: int, k: int, codebook_out, x=None, hist_in=Non
                                      workspace_buf.numel(), _stream(stream))
     _check("gefen_refit_codebook", st)
     return workspace_buf
+
+
+STATIC_MAX_BINS = 4096
+STATIC_MAX_LEVELS = 256
+
+
+def gefen_refit_codebook_static(*, bins: int, k: int, codebook_out, x=None, hist_in=None, hist_out=None,
+                                cell_start_out=None, cost_out=None, stream=None):
+    """gefen_refit_codebook without a workspace: the library's own device
+    array serves as scratch (bins <= 4096, k <= 256).  Nothing is allocated."""
+    if bins > STATIC_MAX_BINS or k > STATIC_MAX_LEVELS:
+        raise GefenError("gefen_refit_codebook_static",
+                         GEFEN_EUNSUPPORTED,
+                         f"bins <= {STATIC_MAX_BINS} and k <= {STATIC_MAX_LEVELS} (got bins={bins}, k={k})")
+    n = x.numel() if x is not None else 0
+    xp = _ptr(x)
+    if x is not None and n == 0:  # an empty input still selects the x path
+        xp = _ptr(codebook_out)
+    st = load().gefen_refit_codebook_static(xp, n, _ptr(hist_in), bins, k, _ptr(codebook_out), _ptr(hist_out),
+                                            _ptr(cell_start_out), _ptr(cost_out), _stream(stream))
+    _check("gefen_refit_codebook_static", st)
 
 
 def gefen_refit_status(workspace_buf, stream=None) -> int:
