@@ -43,7 +43,14 @@ MICRO_N = 1_499_987_968  # 1.5e9 values rounded to whole blocks of 4096
 K = 256
 HP = dict(lr=1e-4, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=0.0)  # Appendix I, Llama
 SEED = 0
-PROFILE = os.path.join(ROOT, "profiles", "step_tile16_llama1p5b.md")
+PROFILE = os.path.join(ROOT, "profiles", "step_stream4k_llama1p5b.md")
+DOMINANT = "k_step_stream<4096> (blocks of p <= 4096, p % 16 == 0, p > 1)"
+
+
+def dominant(p: int) -> bool:
+    """Tensors served by the streamed 4096-element tile kernel, the one that
+    carries most of the step's bytes on this workload."""
+    return p > 1 and p % 16 == 0 and p <= 4096
 
 
 def peaks():
@@ -63,18 +70,19 @@ def step_kernel_source_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def profiled_traffic():
-    """DRAM bytes per launch of the step kernel from the committed ncu summary,
-    or None when it is missing or the kernel source changed since."""
+def profiled_traffic(n_elems: int):
+    """DRAM bytes of one launch of the dominant kernel: the committed ncu
+    summary's bytes per element times the elements one launch processes here;
+    None when the summary is missing or the kernel source changed since."""
     try:
         txt = open(PROFILE).read()
     except OSError:
         return None
     m = re.search(r"source_hash:\s*([0-9a-f]+)", txt)
-    t = re.search(r"traffic_bytes_per_step:\s*([0-9.eE+]+)", txt)
+    t = re.search(r"dram_bytes_per_element:\s*([0-9.eE+]+)", txt)
     if not m or not t or m.group(1) != step_kernel_source_hash():
         return None
-    return float(t.group(1))
+    return float(t.group(1)) * n_elems
 
 
 class Clocks:
@@ -132,9 +140,11 @@ def dist_env():
     return ws, rank, local
 
 
-def launches_per_step(periods, flags_hist: bool) -> int:
+def launches_per_call(periods, flags_hist: bool) -> int:
     """Kernels one gefen_step call launches for these periods (mirrors the
-    library's path classes)."""
+    library's path classes; fewer than 300 tensors per class)."""
+    if not periods:
+        return 0
     cls = set()
     big = 0
     for p in periods:
@@ -198,6 +208,13 @@ def run_gpu(args, world, rank, local):
         boff += s.numel // p
     nblocks = boff
     table = G.tensor_table(entries)
+    # a step is two calls: the tensors of the dominant kernel, then the rest,
+    # so CUDA events time that kernel's launch on its own
+    ent_a = [e for e in entries if dominant(e[2])]
+    ent_b = [e for e in entries if not dominant(e[2])]
+    table_a, table_b = G.tensor_table(ent_a), G.tensor_table(ent_b)
+    n_a = sum(e[1] for e in ent_a)
+    blocks_a = sum(e[1] // e[2] for e in ent_a)
     codes = torch.empty(total, dtype=torch.uint8, device=dev)
     v = torch.zeros(nblocks, dtype=torch.float32, device=dev)
     sc = torch.zeros(nblocks, dtype=torch.float32, device=dev)
@@ -207,6 +224,7 @@ def run_gpu(args, world, rank, local):
 
     # Algorithm 3 on the first gradient: histogram of g / block absmax, DP
     ws = G.workspace(G.gefen_step_workspace_size(table, G.GEFEN_HIST), dev)
+    ws_b = G.workspace(G.gefen_step_workspace_size(table_b, G.GEFEN_HIST), dev)
     rws = G.workspace(G.gefen_refit_workspace_size(BINS, K), dev)
     t0 = time.perf_counter()
     G.gefen_step(table, theta, gpool[0], codes, v, sc, cb, cb, step=1, flags=G.GEFEN_HIST_GRAD_ONLY,
@@ -218,6 +236,7 @@ def run_gpu(args, world, rank, local):
     codes.fill_(zc)
 
     step_events = []   # (start, end) of plain steps
+    dom_events = []    # (start, end) of the dominant kernel's call in plain steps
     refit_events = []  # (step start, step end, dp end)
     state = {"t": 0, "switch": False}
 
@@ -230,14 +249,19 @@ def run_gpu(args, world, rank, local):
         e0 = torch.cuda.Event(enable_timing=True) if timed else None
         e1 = torch.cuda.Event(enable_timing=True) if timed else None
         e2 = torch.cuda.Event(enable_timing=True) if timed and refit else None
+        ea = torch.cuda.Event(enable_timing=True) if timed and not refit else None
         if timed:
             e0.record(stream)
+        flags = G.GEFEN_HIST if refit else 0
         if refit:
             hist.zero_()
-            G.gefen_step(table, theta, g, codes, v, sc, cb, enc, step=t, flags=G.GEFEN_HIST, hist=hist,
-                         workspace_buf=ws, **HP)
-        else:
-            G.gefen_step(table, theta, g, codes, v, sc, cb, enc, step=t, workspace_buf=ws, **HP)
+        G.gefen_step(table_a, theta, g, codes, v, sc, cb, enc, step=t, flags=flags, hist=hist if refit else None,
+                     workspace_buf=ws, **HP)
+        if ea is not None:
+            ea.record(stream)
+            dom_events.append((e0, ea))
+        G.gefen_step(table_b, theta, g, codes, v, sc, cb, enc, step=t, flags=flags, hist=hist if refit else None,
+                     workspace_buf=ws_b, **HP)
         if timed:
             e1.record(stream)
         if state["switch"]:
@@ -276,6 +300,7 @@ def run_gpu(args, world, rank, local):
     time.sleep(0.05)
     ck = clocks.stop()
     G.gefen_step_status(ws)  # raises if a bounded device wait gave up
+    G.gefen_step_status(ws_b)
     elapsed_ms = ev0.elapsed_time(ev1)
     if world > 1:
         import torch.distributed as dist
@@ -291,8 +316,11 @@ def run_gpu(args, world, rank, local):
 
     alg_bytes = 12 * nparams + 16 * nblocks + 8 * K
     hbm, peak_kind = peaks()
-    achieved = alg_bytes / (avg_step_ms * 1e-3) / 1e9
-    traffic = profiled_traffic()
+    # the dominant kernel alone: 12 bytes per parameter and 16 per block
+    dom_ms = statistics.mean([a.elapsed_time(b) for a, b in dom_events]) if dom_events else float("nan")
+    alg_bytes_a = 12 * n_a + 16 * blocks_a
+    achieved = alg_bytes_a / (dom_ms * 1e-3) / 1e9
+    traffic = profiled_traffic(n_a)
 
     # e2e: gradient in from pinned host memory, parameters back, every step
     e2e = None
@@ -300,8 +328,11 @@ def run_gpu(args, world, rank, local):
         e2e = run_e2e(G, table, theta, codes, v, sc, cb, ws, gpool, nparams, stream, args, state, one_step_ctx=(
             hist, cb_new, rws))
 
-    n_launch_plain = launches_per_step(periods, False)
-    n_launch_refit = launches_per_step(periods, True) + 1 + 1 + (K - 1) + 1  # hist + prefix + levels + backtrack
+    per_a = [e[2] for e in ent_a]
+    per_b = [e[2] for e in ent_b]
+    n_launch_plain = launches_per_call(per_a, False) + launches_per_call(per_b, False)
+    # refit steps: one histogram per call, then the DP: prefix, levels 1..K-1 and the last, backtrack
+    n_launch_refit = launches_per_call(per_a, True) + launches_per_call(per_b, True) + 1 + (K - 1) + 1
     nref = len(refit_events)
     launches = (args.steps - nref) * n_launch_plain + nref * n_launch_refit
 
@@ -319,8 +350,11 @@ def run_gpu(args, world, rank, local):
                    "parallelism": "replicas" if world > 1 else "single GPU"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
                      "frac": achieved / hbm, "traffic": traffic,
-                     "kernel": "gefen_step (k_step_tile16 dominant)", "peak_kind": peak_kind,
-                     "alg_bytes_per_step": alg_bytes, "avg_step_ms": avg_step_ms},
+                     "kernel": DOMINANT, "peak_kind": peak_kind,
+                     "alg_bytes_per_launch": alg_bytes_a, "params_per_launch": n_a, "blocks_per_launch": blocks_a,
+                     "avg_launch_ms": dom_ms,
+                     "whole_step": {"alg_bytes": alg_bytes, "avg_ms": avg_step_ms,
+                                    "achieved_gbs": alg_bytes / (avg_step_ms * 1e-3) / 1e9}},
         "step_only": {"value": nparams / (avg_step_ms * 1e-3) / 1e9 if plain_ms else None, "unit": UNIT,
                       "ms": avg_step_ms},
         "refit": {"dp_ms": statistics.mean(dp_ms) if dp_ms else None,

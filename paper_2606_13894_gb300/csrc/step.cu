@@ -11,6 +11,9 @@
 // bf16 g, u8 code read+write).  Every element's write needs its block's final
 // reductions, so the kernels differ by block size:
 //   p == 1                 k_step_p1       elementwise, v and s per element
+//   p % 16 == 0, p <= 8K   k_step_stream   persistent CTAs stream tiles of
+//                                          whole blocks through shared memory
+//                                          (bulk copies): one HBM pass
 //   p % 16 == 0, p <= 16K  k_step_tile16   one CTA holds whole blocks in
 //                                          registers: one HBM pass
 //   other p <= 2048        k_step_generic  the same with scalar accesses
@@ -370,32 +373,57 @@ __global__ void __launch_bounds__(kThreads) k_step_tile16(const __grid_constant_
 }
 
 // ------------------------------------------------ streamed tiles (bulk copy)
-// Persistent CTAs stream tiles of whole blocks (p % 16 == 0, p <= TILE)
-// through a STAGES-deep shared-memory ring: thread 0 issues cp.async.bulk
-// copies of theta, g and codes for tile i+STAGES-1 while every thread works on
-// tile i, and writes theta' and codes' back with bulk stores.  Decoding uses a
-// shared table; encoding maps x = m / s' to its cell of a uniform grid over
-// [-1, 1] whose record holds the number of midpoints below the cell and the next
-// three midpoints, so the nearest level is base + three compares (identical to
-// the binary search, which remains the fallback when a cell holds more than
-// three midpoints).
+// Persistent CTAs stream tiles of whole blocks (p % 16 == 0, p <= TILE).
+// Thread 0 keeps STAGES tiles of g and codes in flight through a ring of
+// shared-memory stages (cp.async.bulk, completion on an mbarrier) and asks L2
+// to prefetch the same tiles' theta.  A warp owns 512 consecutive elements of
+// a tile; lane l owns the four groups of four at 128 j + 4 l (j < 4), so every
+// warp-wide access of theta, g, codes or x is one contiguous run.
+// Theta is read straight from global memory (an L2 hit) and theta' and the
+// new codes are stored straight from registers, so a stage is free again as
+// soon as its tile is decoded.
+//
+// Decoding reads a shared table; encoding maps x = m / s' to its cell of a
+// uniform grid over [-1, 1] whose record holds the number of midpoints below
+// the cell and the next three midpoints, so the nearest level is base + three
+// compares (identical to the binary search, which remains the fallback when a
+// cell holds more than three midpoints).  Both tables are replicated (LUTR,
+// DECR copies, lane l reading copy l % R) so the gathers of one warp spread
+// over more shared-memory banks.
 constexpr int kLutCells = 512;
 constexpr float kLutGuard = 2.384185791015625e-07f;  // 2^-22, below every cell edge
 
+struct TileInfo {
+    int64_t e0;    // first element
+    int64_t bo;    // first block index into v / scale
+    int nelem;
+    int nblk;
+    int p;
+    uint32_t pmagic;  // floor(2^32 / p) + 1: e / p == umulhi(e, pmagic) for e, p < 2^16
+};
+
+template <int LUTR, int DECR>
 struct alignas(16) StreamTables {
-    float4 lut[kLutCells + 2];  // record c+1 for cell c in [-1, kLutCells]
-    float dec[kMaxLevels];
+    float4 lut[(kLutCells + 2) * LUTR];  // copy r of record c+1 (cell c in [-1, kLutCells]) at (c+1) LUTR + r
+    float dec[kMaxLevels * DECR];        // copy r of level c at c DECR + r
     float mid[kMaxLevels + 4];
 };
 
-template <int TILE, int THREADS, int STAGES>
+// Stage layout: [theta f32 (THS only) | g bf16 | codes u8].
+template <int TILE, bool THS>
+struct StageLayout {
+    static constexpr int kG = THS ? 4 * TILE : 0;
+    static constexpr int kC = kG + 2 * TILE;
+    static constexpr int kBytes = kC + TILE;
+};
+
+template <int TILE, int THREADS, int STAGES, int LUTR, int DECR, bool THS>
 struct alignas(128) StreamSmem {
-    unsigned char stage[STAGES][TILE * 7];  // theta f32 | g bf16 | codes u8
-    StreamTables tab;
-    float2 part[TILE / 8];   // per 8-element group (or per warp): (sum g^2, max |m|)
-    float2 blk[TILE / 16];   // per block: (step factor, 1/s')  [grad-only: (-, absmax)]
-    float sold[TILE / 16];   // per block: scale before the step
-    float vold[TILE / 16];   // per block: v before the step
+    unsigned char stage[STAGES][StageLayout<TILE, THS>::kBytes];
+    StreamTables<LUTR, DECR> tab;
+    float2 part[THREADS / 32];  // per warp: (sum g^2, max |m|)
+    float2 blk[TILE / 16];      // per block, irregular shapes: (step factor, 1/s')  [grad-only: (-, absmax)]
+    TileInfo tile[STAGES];      // the tile each stage holds, written by the issuing thread
     unsigned long long bar[STAGES];
 };
 
@@ -430,62 +458,46 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t
                  "l"(src), "r"(bytes), "r"(bar)
                  : "memory");
 }
-__device__ __forceinline__ void bulk_s2g(void* dst, uint32_t src, uint32_t bytes) {
-    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst), "r"(src), "r"(bytes)
-                 : "memory");
+__device__ __forceinline__ void prefetch_l2(const void* src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
 }
-__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void bulk_wait_read_all() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
-__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
-__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
 // Decode table, midpoints (padded with +inf) and the cell records.
-template <int THREADS>
-__device__ __forceinline__ int build_tables(const Ptrs& P, StreamTables& T, bool grad_only) {
+template <int THREADS, int LUTR, int DECR>
+__device__ __forceinline__ int build_tables(const Ptrs& P, StreamTables<LUTR, DECR>& T, bool grad_only) {
     const int t = threadIdx.x;
     if (grad_only) return 0;
-    for (int i = t; i < kMaxLevels + 4; i += THREADS) {
-        if (i < kMaxLevels) T.dec[i] = i < P.k ? P.cb_dec[i] : 0.0f;
-        T.mid[i] = (i < P.k - 1) ? 0.5f * (P.cb_enc[i] + P.cb_enc[i + 1]) : INFINITY;
+    for (int i = t; i < kMaxLevels * DECR; i += THREADS) {
+        const int c = i / DECR;
+        T.dec[i] = c < P.k ? P.cb_dec[c] : 0.0f;
     }
+    for (int i = t; i < kMaxLevels + 4; i += THREADS)
+        T.mid[i] = (i < P.k - 1) ? 0.5f * (P.cb_enc[i] + P.cb_enc[i + 1]) : INFINITY;
     __syncthreads();
     int bad = 0;
     // cell(x) = floor(fma(x, G/2, G/2)) is within 2^-24 of exact in x: each
     // record counts the midpoints below its cell minus a 2^-22 guard and holds
     // the next three; its cell plus the guard on both sides may hold at most
     // three midpoints, or the binary search is used instead.
-    for (int c = t - 1; c <= kLutCells; c += THREADS) {
+    for (int i = t; i < kLutCells + 2; i += THREADS) {
+        const int c = i - 1;
         const float lo = -1.0f + 2.0f * static_cast<float>(c) / kLutCells - kLutGuard;
         const float hi = -1.0f + 2.0f * static_cast<float>(c + 1) / kLutCells + kLutGuard;
         const int base = level_search(T.mid, lo);
         const int upto = level_search(T.mid, hi);
         bad |= (upto - base > 3);
-        T.lut[c + 1] = make_float4(__int_as_float(base), T.mid[base], T.mid[base + 1], T.mid[base + 2]);
+        const float4 rec = make_float4(__int_as_float(base), T.mid[base], T.mid[base + 1], T.mid[base + 2]);
+#pragma unroll
+        for (int r = 0; r < LUTR; ++r) T.lut[i * LUTR + r] = rec;
     }
     return bad;
 }
 
-__device__ __forceinline__ int encode_lut(const StreamTables& T, bool lut_ok, float x) {
-    if (lut_ok) {
-        int c = __float2int_rd(__fmaf_rn(x, 0.5f * kLutCells, 0.5f * kLutCells));
-        c = min(max(c, -1), kLutCells);
-        const float4 r = T.lut[c + 1];
-        return __float_as_int(r.x) + (r.y < x) + (r.z < x) + (r.w < x);
-    }
-    return level_search(T.mid, x);
-}
-
-struct TileInfo {
-    int64_t e0;    // first element
-    int64_t bo;    // first block index into v / scale
-    int nelem;
-    int nblk;
-    int p;
-    uint32_t pmagic;  // floor(2^32 / p) + 1: e / p == umulhi(e, pmagic) for e, p < 2^16
-};
-
-__device__ __forceinline__ TileInfo tile_info(const Launch& L, int64_t unit) {
-    const Seg& S = L.seg[find_seg(L, unit)];
+// The issuing thread walks the segment table forward: a CTA's tiles come in
+// increasing unit order, so its segment cursor only grows.
+__device__ __forceinline__ TileInfo tile_info(const Launch& L, int64_t unit, int& seg) {
+    while (seg + 1 < L.nseg && L.seg[seg + 1].unit_begin <= unit) ++seg;
+    const Seg& S = L.seg[seg];
     const int64_t p = S.period;
     const int64_t blk0 = (unit - S.unit_begin) * S.per_unit;
     TileInfo ti;
@@ -505,229 +517,346 @@ __device__ __forceinline__ bool tile_fits(const TileInfo& ti) {
     return ti.nelem > 0 && ti.nelem <= TILE && (ti.nelem & 15) == 0;
 }
 
-template <int TILE, int MODE>
-__device__ __forceinline__ void issue_tile(unsigned char* stage, uint32_t bar, const TileInfo& ti, const Ptrs& P) {
+// Publishes the tile's descriptor in its stage and starts its copies.
+template <int TILE, int MODE, bool THS, typename Smem>
+__device__ __forceinline__ void issue_tile(Smem& sm, int s, const TileInfo& ti, const Ptrs& P) {
+    using SL = StageLayout<TILE, THS>;
+    sm.tile[s] = ti;
     if (!tile_fits<TILE>(ti)) return;  // never copied; the consumer stops before waiting on it
     const uint32_t n = static_cast<uint32_t>(ti.nelem);
+    const uint32_t bar = smem_u32(&sm.bar[s]);
+    unsigned char* st = sm.stage[s];
     if (MODE == kGradOnly) {
         mbar_expect_tx(bar, 2u * n);
-        bulk_g2s(smem_u32(stage + 4 * TILE), P.grads + ti.e0, 2u * n, bar);
+        bulk_g2s(smem_u32(st + SL::kG), P.grads + ti.e0, 2u * n, bar);
     } else {
-        mbar_expect_tx(bar, 7u * n);
-        bulk_g2s(smem_u32(stage), P.params + ti.e0, 4u * n, bar);
-        bulk_g2s(smem_u32(stage + 4 * TILE), P.grads + ti.e0, 2u * n, bar);
-        bulk_g2s(smem_u32(stage + 6 * TILE), P.codes + ti.e0, n, bar);
+        mbar_expect_tx(bar, (THS ? 7u : 3u) * n);
+        if (THS) bulk_g2s(smem_u32(st), P.params + ti.e0, 4u * n, bar);
+        bulk_g2s(smem_u32(st + SL::kG), P.grads + ti.e0, 2u * n, bar);
+        bulk_g2s(smem_u32(st + SL::kC), P.codes + ti.e0, n, bar);
+        if (!THS) prefetch_l2(P.params + ti.e0, 4u * n);
     }
 }
 
-template <int TILE, int THREADS, int STAGES, int MODE, int MINB>
-__global__ void __launch_bounds__(THREADS, MINB) k_step_stream(const __grid_constant__ Launch L, const Ptrs P, int* err) {
-    using Smem = StreamSmem<TILE, THREADS, STAGES>;
-    // each thread owns one group of 8 consecutive elements of the tile
-    static_assert(TILE == 8 * THREADS && THREADS >= TILE / 16 && THREADS % 32 == 0, "tile shape");
-    extern __shared__ __align__(128) unsigned char smem_raw[];
-    Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const HP& hp = L.hp;
-    const int64_t G = gridDim.x;
-
-    if (tid == 0) {
-        for (int s = 0; s < STAGES; ++s) mbar_init(smem_u32(&sm.bar[s]), 1u);
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+// Block state (s and v before the step) of the blocks of the thread's NG
+// groups, whose first elements are eb + 128 j.
+template <int NG>
+__device__ __forceinline__ void load_state(const Ptrs& P, const TileInfo& ti, int eb, float (&s)[NG], float (&v)[NG]) {
+    if (ti.p > 65535) return;              // only a tile that does not fit; never processed
+    if (ti.p % (128 * NG) == 0) {          // one block per warp slice
+        if (eb < ti.nelem) {
+            const int64_t bi = ti.bo + __umulhi(static_cast<uint32_t>(eb), ti.pmagic);
+            const float s0 = P.scale[bi], v0 = P.v[bi];
+#pragma unroll
+            for (int j = 0; j < NG; ++j) { s[j] = s0; v[j] = v0; }
+        }
+        return;
     }
-    const int bad = build_tables<THREADS>(P, sm.tab, MODE == kGradOnly);
-    const bool lut_ok = !__syncthreads_or(bad);
-    const int zero_code = (MODE != kGradOnly) ? level_search(sm.tab.mid, 0.0f) : 0;
-
-    if (tid == 0) {
-        for (int s = 0; s < STAGES - 1; ++s) {
-            const int64_t u = blockIdx.x + s * G;
-            if (u < L.nunits) issue_tile<TILE, MODE>(sm.stage[s], smem_u32(&sm.bar[s]), tile_info(L, u), P);
+#pragma unroll
+    for (int j = 0; j < NG; ++j) {
+        const int e = eb + 128 * j;
+        if (e < ti.nelem) {
+            const int64_t bi = ti.bo + __umulhi(static_cast<uint32_t>(e), ti.pmagic);
+            s[j] = P.scale[bi];
+            v[j] = P.v[bi];
         }
     }
-    // block state of the first tile; later tiles' state is loaded one tile ahead
-    float r_sold = 0.0f, r_vold = 0.0f;
-    if (MODE != kGradOnly && blockIdx.x < L.nunits) {
-        const TileInfo t0 = tile_info(L, blockIdx.x);
-        if (tid < t0.nblk) { r_sold = P.scale[t0.bo + tid]; r_vold = P.v[t0.bo + tid]; }
+}
+
+__device__ __forceinline__ void butterfly(float& s2, float& mx, int lanes) {
+    for (int o = lanes >> 1; o > 0; o >>= 1) {
+        s2 += __shfl_xor_sync(0xffffffffu, s2, o);
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
     }
+}
+
+// 0xFFFFFFFF if a < b else 0 (one compare that yields an integer mask)
+__device__ __forceinline__ uint32_t lt_mask(float a, float b) {
+    uint32_t r;
+    asm("set.lt.u32.f32 %0, %1, %2;" : "=r"(r) : "f"(a), "f"(b));
+    return r;
+}
+
+// Nearest levels of four values, packed as four code bytes.  With the cell
+// records (LUT): |x| <= 1 up to rounding (x = m / max|m|, or 0 for a zero
+// block), so the record index floor(256 x + 257) lies in [0, 513].  The floor
+// is one round-down fma against 1.5 * 2^23, where the float grid is the
+// integers: y = floor(256 x + 257) + 1.5 * 2^23 exactly, and the index is the
+// bit pattern of y minus that of 1.5 * 2^23.  The unsigned clamp keeps a NaN
+// or a corrupted value inside the table.
+template <bool LUT, int LUTR, int DECR>
+__device__ __forceinline__ uint32_t encode4(const StreamTables<LUTR, DECR>& T, int copy, const float (&x)[4]) {
+    constexpr float kMagic = 12582912.0f;  // 1.5 * 2^23, bits 0x4B400000
+    uint32_t c[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        if (LUT) {
+            const float y = __fmaf_rd(x[i], 0.5f * kLutCells, 0.5f * kLutCells + 1.0f + kMagic);
+            const uint32_t r = static_cast<uint32_t>(__float_as_int(y)) - 0x4B400000u;
+            const float4 rec = T.lut[min(r, static_cast<uint32_t>(kLutCells + 1)) * LUTR + copy];
+            c[i] = static_cast<uint32_t>(__float_as_int(rec.x)) - lt_mask(rec.y, x[i]) - lt_mask(rec.z, x[i]) -
+                   lt_mask(rec.w, x[i]);
+        } else {
+            c[i] = static_cast<uint32_t>(level_search(T.mid, x[i]));
+        }
+    }
+    return __byte_perm(__byte_perm(c[0], c[1], 0x0040u), __byte_perm(c[2], c[3], 0x0040u), 0x5410u);
+}
+
+// One tile of the streamed step.  FULL: every group of the tile is live (the
+// tile holds TILE elements), so no group needs a bounds predicate.
+template <int TILE, int THREADS, int LUTR, int DECR, int MODE, bool THS, bool LUT, bool FULL, typename Smem>
+__device__ __forceinline__ void stream_tile(Smem& sm, const Ptrs& P, const HP& hp, const TileInfo& ti,
+                                            unsigned char* st, int eb, const float (&r_s)[4], const float (&r_v)[4]) {
+    using SL = StageLayout<TILE, THS>;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int lut_copy = lane % LUTR, dec_copy = lane % DECR;
+    const int p = ti.p;
+    const float rp = __frcp_rn(static_cast<float>(p));
+    bool live[4];
+    int blk[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        const int e = eb + 128 * j;
+        live[j] = FULL || e < ti.nelem;
+        blk[j] = static_cast<int>(__umulhi(static_cast<uint32_t>(e), ti.pmagic));
+    }
+    float* thp = P.params + ti.e0 + eb;  // group j at + 128 j
+    float4 th[4];  // theta from global memory is loaded early; from the stage, just before use
+    if (MODE != kGradOnly && !THS) {
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+            if (live[j]) th[j] = __ldcs(reinterpret_cast<const float4*>(thp + 128 * j));
+    }
+
+    // phase 1: decode m, partials per group of four
+    float m[16], g2[4], mx[4];
+    const float* dec = sm.tab.dec + dec_copy;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        g2[j] = 0.0f;
+        mx[j] = 0.0f;
+        const int e = eb + 128 * j;
+        const uint2 gw = live[j] ? *reinterpret_cast<const uint2*>(st + SL::kG + 2 * e) : make_uint2(0u, 0u);
+        const float g[4] = {bf16_lo(gw.x), bf16_hi(gw.x), bf16_lo(gw.y), bf16_hi(gw.y)};
+        if (MODE == kGradOnly) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                m[4 * j + i] = g[i];
+                mx[j] = fmaxf(mx[j], fabsf(g[i]));
+            }
+        } else {
+            const uint32_t cw = live[j] ? *reinterpret_cast<const uint32_t*>(st + SL::kC + e) : 0u;
+            const float b1s = hp.beta1 * r_s[j];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const uint32_t c = __byte_perm(cw, 0u, 0x4440u + i);
+                const float mm = fmaf(hp.omb1, g[i], b1s * dec[c * DECR]);
+                m[4 * j + i] = mm;
+                g2[j] = fmaf(g[i], g[i], g2[j]);
+                mx[j] = fmaxf(mx[j], fabsf(mm));
+            }
+        }
+    }
+
+    // block reductions: every lane holding a block ends with the same sums
+    // (butterflies are exact under commutation; lists of partials are summed
+    // in one fixed order), so each derives the block's factors
+    float fac[4], inv[4];  // grad-only: inv = max |g|
+    auto finish = [&](float s2, float sx, float v_old, int64_t bi, bool writer, float& f, float& iv) {
+        if (MODE == kGradOnly) {
+            iv = sx;
+            f = 0.0f;
+        } else {
+            const float vn = fmaf(hp.beta2, v_old, hp.omb2 * (s2 * rp));
+            f = hp.lr_bc1 * __frcp_rn(sqrtf(vn * hp.inv_bc2) + hp.eps);
+            iv = sx > 0.0f ? __frcp_rn(sx) : 0.0f;
+            if (writer) {
+                P.v[bi] = vn;
+                P.scale[bi] = sx;
+            }
+        }
+    };
+    if ((p & 511) == 0) {
+        // a warp's 512 elements lie in one block
+        float s2 = (g2[0] + g2[1]) + (g2[2] + g2[3]);
+        float sx = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+        butterfly(s2, sx, 32);
+        const int nw = p >> 9;  // warps per block
+        if (nw > 1) {
+            if (lane == 0) sm.part[warp] = make_float2(s2, sx);
+            __syncthreads();
+            const int w0 = warp - warp % nw;
+            s2 = 0.0f;
+            sx = 0.0f;
+            for (int t = 0; t < nw; ++t) {
+                const float2 pp = sm.part[w0 + t];
+                s2 += pp.x;
+                sx = fmaxf(sx, pp.y);
+            }
+        }
+        finish(s2, sx, r_v[0], ti.bo + blk[0], live[0] && lane == 0 && warp % nw == 0, fac[0], inv[0]);
+#pragma unroll
+        for (int j = 1; j < 4; ++j) { fac[j] = fac[0]; inv[j] = inv[0]; }
+    } else if (p == 256) {
+        // groups 0,1 and 2,3 form one block each
+        float s0 = g2[0] + g2[1], x0 = fmaxf(mx[0], mx[1]);
+        float s1 = g2[2] + g2[3], x1 = fmaxf(mx[2], mx[3]);
+        butterfly(s0, x0, 32);
+        butterfly(s1, x1, 32);
+        finish(s0, x0, r_v[0], ti.bo + blk[0], live[0] && lane == 0, fac[0], inv[0]);
+        finish(s1, x1, r_v[2], ti.bo + blk[2], live[2] && lane == 0, fac[2], inv[2]);
+        fac[1] = fac[0]; inv[1] = inv[0];
+        fac[3] = fac[2]; inv[3] = inv[2];
+    } else if ((p & (p - 1)) == 0) {
+        // p in {16, 32, 64, 128}: a block spans p/4 lanes of one group
+        const int lanes = p >> 2;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            butterfly(g2[j], mx[j], lanes);
+            finish(g2[j], mx[j], r_v[j], ti.bo + blk[j], live[j] && (lane & (lanes - 1)) == 0, fac[j], inv[j]);
+        }
+    } else {
+        // any other shape: each group's partial goes over the thread's own
+        // (already decoded) g bytes of that group, then one warp per block
+        float2* part4 = reinterpret_cast<float2*>(st + SL::kG);  // partial of group e/4 at byte 2e of g
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+            if (live[j]) part4[(eb + 128 * j) >> 2] = make_float2(g2[j], mx[j]);
+        // the stage is refilled by bulk copies (async proxy) after these writes
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        __syncthreads();
+        const int q4 = p >> 2;  // groups per block
+        for (int bb = warp; bb < ti.nblk; bb += THREADS / 32) {
+            float s2 = 0.0f, sx = 0.0f;
+            for (int t = lane; t < q4; t += 32) {
+                const float2 pp = part4[bb * q4 + t];
+                s2 += pp.x;
+                sx = fmaxf(sx, pp.y);
+            }
+            s2 = warp_sum(s2);
+            sx = warp_max(sx);
+            if (lane == 0) {
+                float f = 0.0f, iv = 0.0f;
+                finish(s2, sx, MODE == kGradOnly ? 0.0f : P.v[ti.bo + bb], ti.bo + bb, true, f, iv);
+                sm.blk[bb] = make_float2(f, iv);
+            }
+        }
+        __syncthreads();
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const float2 bs = live[j] ? sm.blk[blk[j]] : make_float2(0.0f, 0.0f);
+            fac[j] = bs.x;
+            inv[j] = bs.y;
+        }
+    }
+
+    // phase 2: theta', the new codes (and x for the histogram), stored
+    // straight from registers.  A zero block (inv = 0) encodes x = 0, the
+    // level nearest 0, and stages NaN for the histogram.
+    uint8_t* cdp = P.codes + ti.e0 + eb;
+    float* xsp = (MODE != kPlain) ? P.xstage + ti.e0 + eb : nullptr;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        if (!live[j]) continue;
+        float x[4];
+        if (MODE == kGradOnly) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                x[i] = inv[j] > 0.0f ? __fdiv_rn(m[4 * j + i], inv[j]) : __int_as_float(0x7fffffff);
+        } else {
+            float4 t = THS ? *reinterpret_cast<const float4*>(st + 4 * (eb + 128 * j)) : th[j];
+            t.x = fmaf(-fac[j], m[4 * j], hp.decay * t.x);
+            t.y = fmaf(-fac[j], m[4 * j + 1], hp.decay * t.y);
+            t.z = fmaf(-fac[j], m[4 * j + 2], hp.decay * t.z);
+            t.w = fmaf(-fac[j], m[4 * j + 3], hp.decay * t.w);
+            __stcs(reinterpret_cast<float4*>(thp + 128 * j), t);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) x[i] = m[4 * j + i] * inv[j];
+            __stcs(reinterpret_cast<unsigned int*>(cdp + 128 * j), encode4<LUT>(sm.tab, lut_copy, x));
+            if (MODE == kHist) {
+#pragma unroll
+                for (int i = 0; i < 4; ++i) x[i] = inv[j] > 0.0f ? x[i] : __int_as_float(0x7fffffff);
+            }
+        }
+        if (MODE != kPlain) __stcs(reinterpret_cast<float4*>(xsp + 128 * j), make_float4(x[0], x[1], x[2], x[3]));
+    }
+}
+
+template <int TILE, int THREADS, int STAGES, int LUTR, int DECR, int MODE, bool THS, bool LUT, typename Smem>
+__device__ __forceinline__ void stream_loop(Smem& sm, const Launch& L, const Ptrs& P, int* err, int seg) {
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int64_t G = gridDim.x;
+    const int eb = warp * 512 + lane * 4;  // first element of the thread's group 0 within a tile
+
+    float r_s[4] = {0.0f, 0.0f, 0.0f, 0.0f}, r_v[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    if (MODE != kGradOnly && blockIdx.x < L.nunits) load_state<4>(P, sm.tile[0], eb, r_s, r_v);
 
     for (int it = 0;; ++it) {
         const int64_t u = blockIdx.x + static_cast<int64_t>(it) * G;
         if (u >= L.nunits) break;
         const int s = it % STAGES;
         const uint32_t parity = static_cast<uint32_t>((it / STAGES) & 1);
-        const TileInfo ti = tile_info(L, u);
-        if (!tile_fits<TILE>(ti)) {
-            // a tile the host planned too large: nothing was copied for it.
-            // Wait (bounded) for the copies already issued for later tiles,
-            // flag the error and stop.
-            for (int j = 1; j < STAGES; ++j) {
+        const TileInfo ti = sm.tile[s];
+        const bool fits = tile_fits<TILE>(ti);
+        const bool ok = fits ? mbar_wait(smem_u32(&sm.bar[s]), parity) : true;
+        if (__syncthreads_or(!fits || !ok)) {
+            // A tile the host planned too large (nothing was copied for it) or
+            // a copy that never completed: wait, bounded, for the copies still
+            // in flight, flag the error and stop.
+            for (int j = fits ? 0 : 1; j < STAGES; ++j) {
                 const int64_t uj = u + static_cast<int64_t>(j) * G;
-                if (uj >= L.nunits || !tile_fits<TILE>(tile_info(L, uj))) continue;
+                if (uj >= L.nunits || !tile_fits<TILE>(sm.tile[(it + j) % STAGES])) continue;
                 mbar_wait(smem_u32(&sm.bar[(it + j) % STAGES]), static_cast<uint32_t>(((it + j) / STAGES) & 1));
             }
-            if (tid == 0) atomicExch(err, 2);
+            if (tid == 0) atomicExch(err, fits ? 1 : 2);
             break;
         }
-        if (MODE != kGradOnly) {
-            if (tid < ti.nblk) { sm.sold[tid] = r_sold; sm.vold[tid] = r_vold; }
-            if (u + G < L.nunits) {
-                const TileInfo tn = tile_info(L, u + G);
-                if (tid < tn.nblk) { r_sold = P.scale[tn.bo + tid]; r_vold = P.v[tn.bo + tid]; }
-            }
-        }
-        const bool ok = mbar_wait(smem_u32(&sm.bar[s]), parity);
-        if (__syncthreads_or(!ok)) {
-            if (tid == 0) atomicExch(err, 1);
-            break;
-        }
-        unsigned char* st = sm.stage[s];
-        float* sth = reinterpret_cast<float*>(st);
-        const uint16_t* sg = reinterpret_cast<const uint16_t*>(st + 4 * TILE);
-        uint8_t* sc = st + 6 * TILE;
-        const int q = ti.p >> 3;  // 8-element groups per block (p % 16 == 0)
-        const float pf = static_cast<float>(ti.p);
-        // a block whose groups all sit in one warp finishes in phase 1
-        const bool seg = (q <= 32) && ((32 % q) == 0);
-        const bool warp_part = !seg && (q % 32 == 0);
-        auto finish = [&](int b, float g2, float mx) {
-            if (MODE == kGradOnly) {
-                sm.blk[b] = make_float2(0.0f, mx);
-            } else {
-                const float vn = fmaf(hp.beta2, sm.vold[b], hp.omb2 * (g2 / pf));
-                P.v[ti.bo + b] = vn;
-                P.scale[ti.bo + b] = mx;
-                const float fac = hp.lr_bc1 / (sqrtf(vn * hp.inv_bc2) + hp.eps);
-                sm.blk[b] = make_float2(fac, mx > 0.0f ? 1.0f / mx : 0.0f);
-            }
-        };
+        // block state of the next tile, one tile ahead (its descriptor was
+        // published before the barrier above)
+        float n_s[4] = {0.0f, 0.0f, 0.0f, 0.0f}, n_v[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+        if (MODE != kGradOnly && u + G < L.nunits) load_state<4>(P, sm.tile[(it + 1) % STAGES], eb, n_s, n_v);
 
-        // phase 1: decode m, partials over the thread's 8 elements
-        const int e = tid * 8;
-        const bool live = e < ti.nelem;
-        const int b = static_cast<int>(__umulhi(static_cast<uint32_t>(e), ti.pmagic));
-        float m[8];
-        float g2 = 0.0f, mx = 0.0f;
-        if (live) {
-            const uint4 gw = *reinterpret_cast<const uint4*>(sg + e);
-            const uint32_t gws[4] = {gw.x, gw.y, gw.z, gw.w};
-            if (MODE == kGradOnly) {
-#pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    m[2 * j] = bf16_lo(gws[j]);
-                    m[2 * j + 1] = bf16_hi(gws[j]);
-                }
-#pragma unroll
-                for (int j = 0; j < 8; ++j) mx = fmaxf(mx, fabsf(m[j]));
-            } else {
-                const uint2 cw = *reinterpret_cast<const uint2*>(sc + e);
-                const float b1s = hp.beta1 * sm.sold[b];
-#pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    const float g = (j & 1) ? bf16_hi(gws[j >> 1]) : bf16_lo(gws[j >> 1]);
-                    const uint32_t c = ((j < 4 ? cw.x : cw.y) >> (8 * (j & 3))) & 0xFFu;
-                    const float mm = fmaf(hp.omb1, g, b1s * sm.tab.dec[c]);
-                    m[j] = mm;
-                    g2 = fmaf(g, g, g2);
-                    mx = fmaxf(mx, fabsf(mm));
-                }
-            }
-        }
-        if (seg) {
-            for (int o = q >> 1; o > 0; o >>= 1) {
-                g2 += __shfl_xor_sync(0xffffffffu, g2, o);
-                mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-            }
-            if (live && (tid % q) == 0) finish(b, g2, mx);
-        } else if (warp_part) {
-            g2 = warp_sum(g2);
-            mx = warp_max(mx);
-            if (lane == 0) sm.part[tid >> 5] = make_float2(g2, mx);
-        } else {
-            sm.part[tid] = make_float2(g2, mx);
-        }
-        __syncthreads();
-        if (!seg) {
-            // remaining block reductions over the stored partials (fixed order)
-            const int per = warp_part ? (q >> 5) : q;
-            for (int bb = warp; bb < ti.nblk; bb += THREADS / 32) {
-                float s2 = 0.0f, sx = 0.0f;
-                for (int t = lane; t < per; t += 32) {
-                    const float2 pp = sm.part[bb * per + t];
-                    s2 += pp.x;
-                    sx = fmaxf(sx, pp.y);
-                }
-                s2 = warp_sum(s2);
-                sx = warp_max(sx);
-                if (lane == 0) finish(bb, s2, sx);
-            }
-            __syncthreads();
-        }
+        if (ti.nelem == TILE)
+            stream_tile<TILE, THREADS, LUTR, DECR, MODE, THS, LUT, true>(sm, P, L.hp, ti, sm.stage[s], eb, r_s, r_v);
+        else
+            stream_tile<TILE, THREADS, LUTR, DECR, MODE, THS, LUT, false>(sm, P, L.hp, ti, sm.stage[s], eb, r_s, r_v);
 
-        // phase 2: update and re-encode into the stage, x to the staging buffer
-        if (live) {
-            const float2 bs = sm.blk[b];
-            float x[8];
-            if (MODE == kGradOnly) {
-#pragma unroll
-                for (int j = 0; j < 8; ++j) x[j] = bs.y > 0.0f ? __fdiv_rn(m[j], bs.y) : __int_as_float(0x7fffffff);
-            } else {
-                float4* tp = reinterpret_cast<float4*>(sth + e);
-                float4 t0 = tp[0], t1 = tp[1];
-                t0.x = fmaf(-bs.x, m[0], hp.decay * t0.x);
-                t0.y = fmaf(-bs.x, m[1], hp.decay * t0.y);
-                t0.z = fmaf(-bs.x, m[2], hp.decay * t0.z);
-                t0.w = fmaf(-bs.x, m[3], hp.decay * t0.w);
-                t1.x = fmaf(-bs.x, m[4], hp.decay * t1.x);
-                t1.y = fmaf(-bs.x, m[5], hp.decay * t1.y);
-                t1.z = fmaf(-bs.x, m[6], hp.decay * t1.z);
-                t1.w = fmaf(-bs.x, m[7], hp.decay * t1.w);
-                tp[0] = t0;
-                tp[1] = t1;
-                uint32_t w0 = 0, w1 = 0;
-                if (bs.y > 0.0f) {
-#pragma unroll
-                    for (int j = 0; j < 8; ++j) {
-                        x[j] = m[j] * bs.y;
-                        const uint32_t c = static_cast<uint32_t>(encode_lut(sm.tab, lut_ok, x[j]));
-                        if (j < 4) w0 |= c << (8 * j); else w1 |= c << (8 * (j - 4));
-                    }
-                } else {
-                    const uint32_t z = static_cast<uint32_t>(zero_code) * 0x01010101u;
-                    w0 = w1 = z;
-#pragma unroll
-                    for (int j = 0; j < 8; ++j) x[j] = __int_as_float(0x7fffffff);
-                }
-                *reinterpret_cast<uint2*>(sc + e) = make_uint2(w0, w1);
-            }
-            if (MODE != kPlain) {
-                float4* xs = reinterpret_cast<float4*>(P.xstage + ti.e0 + e);
-                __stcs(xs, make_float4(x[0], x[1], x[2], x[3]));
-                __stcs(xs + 1, make_float4(x[4], x[5], x[6], x[7]));
-            }
-        }
-        if (MODE != kGradOnly) fence_proxy_async();
+        // every thread is done with stage s: refill it with tile it + STAGES
         __syncthreads();
         if (tid == 0) {
-            if (MODE != kGradOnly) {
-                const uint32_t n = static_cast<uint32_t>(ti.nelem);
-                bulk_s2g(P.params + ti.e0, smem_u32(sth), 4u * n);
-                bulk_s2g(P.codes + ti.e0, smem_u32(sc), n);
-            }
-            bulk_commit();
-            // Refill the stage tile it-1 used with tile it+STAGES-1.  Its store
-            // was committed an iteration ago: wait until only this tile's
-            // store may still be reading shared memory.
-            const int64_t un = u + static_cast<int64_t>(STAGES - 1) * G;
-            if (un < L.nunits) {
-                asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
-                const int sn = (it + STAGES - 1) % STAGES;
-                issue_tile<TILE, MODE>(sm.stage[sn], smem_u32(&sm.bar[sn]), tile_info(L, un), P);
-            }
+            const int64_t un = u + static_cast<int64_t>(STAGES) * G;
+            if (un < L.nunits) issue_tile<TILE, MODE, THS>(sm, s, tile_info(L, un, seg), P);
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j) { r_s[j] = n_s[j]; r_v[j] = n_v[j]; }
+    }
+}
+
+template <int TILE, int THREADS, int STAGES, int LUTR, int DECR, bool THS, int MODE, int MINB>
+__global__ void __launch_bounds__(THREADS, MINB) k_step_stream(const __grid_constant__ Launch L, const Ptrs P, int* err) {
+    using Smem = StreamSmem<TILE, THREADS, STAGES, LUTR, DECR, THS>;
+    static_assert(TILE == 16 * THREADS && THREADS % 32 == 0 && STAGES >= 2, "tile shape");
+    static_assert(32 % LUTR == 0 && 32 % DECR == 0, "table copies");
+    extern __shared__ __align__(128) unsigned char smem_raw[];
+    Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
+    const int64_t G = gridDim.x;
+    int seg = 0;  // the issuing thread's cursor into L.seg
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) mbar_init(smem_u32(&sm.bar[s]), 1u);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        for (int s = 0; s < STAGES; ++s) {
+            const int64_t u = blockIdx.x + s * G;
+            if (u < L.nunits) issue_tile<TILE, MODE, THS>(sm, s, tile_info(L, u, seg), P);
         }
     }
-    if (tid == 0) bulk_wait_all();
+    const int bad = build_tables<THREADS>(P, sm.tab, MODE == kGradOnly);
+    const bool lut_ok = !__syncthreads_or(bad);
+    if (MODE != kGradOnly && lut_ok)
+        stream_loop<TILE, THREADS, STAGES, LUTR, DECR, MODE, THS, true>(sm, L, P, err, seg);
+    else
+        stream_loop<TILE, THREADS, STAGES, LUTR, DECR, MODE, THS, false>(sm, L, P, err, seg);
 }
 
 // ------------------------------------------- generic p <= 2048 (scalar)
@@ -1043,10 +1172,19 @@ __global__ void __launch_bounds__(kThreads) k_big_apply(const __grid_constant__ 
 // ------------------------------------------------------------- host side
 enum PathClass { kP1 = 0, kS4K, kS8K, kT16V4, kGeneric, kBigAligned, kBigUnaligned, kNumClasses };
 
-// p <= 4096: two 512-thread CTAs per SM, 3-stage rings of 28 KB tiles;
-// p <= 8192: one 1024-thread CTA per SM, 3-stage ring of 56 KB tiles
-constexpr int kS4KTile = 4096, kS4KThreads = 512, kS4KStages = 3, kS4KMinBlocks = 2;
-constexpr int kS8KTile = 8192, kS8KThreads = 1024, kS8KStages = 3, kS8KMinBlocks = 1;
+template <int TILE_, int THREADS_, int STAGES_, int LUTR_, int DECR_, bool THS_, int MINB_>
+struct StreamCfg {
+    static constexpr int TILE = TILE_, THREADS = THREADS_, STAGES = STAGES_, LUTR = LUTR_, DECR = DECR_, MINB = MINB_;
+    static constexpr bool THS = THS_;
+};
+// p <= 4096: two 256-thread CTAs per SM, 3-stage rings of 12 KB tiles (g,
+// codes; theta read from global memory), cell records in 8 copies and the
+// decode table in 8;
+// p <= 8192: one 512-thread CTA per SM, a 2-stage ring of 56 KB tiles
+// (theta staged too), cell records in 8 copies and the decode table in 32.
+using S4KCfg = StreamCfg<4096, 256, 3, 8, 8, false, 2>;
+using S8KCfg = StreamCfg<8192, 512, 2, 8, 32, true, 1>;
+constexpr int kS4KTile = S4KCfg::TILE, kS8KTile = S8KCfg::TILE;
 
 PathClass classify(int64_t p) {
     if (p == 1) return kP1;
@@ -1175,24 +1313,24 @@ cudaError_t launch_class(K kernel, Launch& L, const std::vector<int>& ids, const
     return cudaSuccess;
 }
 
-template <int TILE, int THREADS, int STAGES, int MINB, int MODE>
+template <typename C, int MODE>
 cudaError_t launch_stream(Launch& L, const std::vector<int>& ids, const gefen_tensor_t* t, PathClass c,
                           const Ptrs& P, int* err, cudaStream_t st) {
-    auto kern = k_step_stream<TILE, THREADS, STAGES, MODE, MINB>;
-    const int smem = static_cast<int>(sizeof(StreamSmem<TILE, THREADS, STAGES>));
+    auto kern = k_step_stream<C::TILE, C::THREADS, C::STAGES, C::LUTR, C::DECR, C::THS, MODE, C::MINB>;
+    const int smem = static_cast<int>(sizeof(StreamSmem<C::TILE, C::THREADS, C::STAGES, C::LUTR, C::DECR, C::THS>));
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
     if (e != cudaSuccess) return e;
     int per_sm = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, THREADS, smem);
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, C::THREADS, smem);
     if (e != cudaSuccess) return e;
     const int64_t cap = static_cast<int64_t>(std::max(1, per_sm)) * device_sm_count();
     return launch_class(
         [&](Launch& LL, int64_t u) {
-            kern<<<dim3(static_cast<unsigned>(std::min(u, cap))), THREADS, smem, st>>>(LL, P, err);
+            kern<<<dim3(static_cast<unsigned>(std::min(u, cap))), C::THREADS, smem, st>>>(LL, P, err);
         },
-        L, ids, t, c, TILE);
+        L, ids, t, c, C::TILE);
 }
 
 template <int MODE>
@@ -1201,9 +1339,9 @@ cudaError_t run_step(const Plan& pl, const gefen_tensor_t* t, Launch& L, const P
     e = launch_class([&](Launch& LL, int64_t u) { k_step_p1<MODE><<<dim3(u), kThreads, 0, st>>>(LL, P); },
                      L, pl.idx[kP1], t, kP1);
     if (e != cudaSuccess) return e;
-    e = launch_stream<kS4KTile, kS4KThreads, kS4KStages, kS4KMinBlocks, MODE>(L, pl.idx[kS4K], t, kS4K, P, err, st);
+    e = launch_stream<S4KCfg, MODE>(L, pl.idx[kS4K], t, kS4K, P, err, st);
     if (e != cudaSuccess) return e;
-    e = launch_stream<kS8KTile, kS8KThreads, kS8KStages, kS8KMinBlocks, MODE>(L, pl.idx[kS8K], t, kS8K, P, err, st);
+    e = launch_stream<S8KCfg, MODE>(L, pl.idx[kS8K], t, kS8K, P, err, st);
     if (e != cudaSuccess) return e;
     e = launch_class([&](Launch& LL, int64_t u) { k_step_tile16<4, MODE><<<dim3(u), kThreads, 0, st>>>(LL, P); },
                      L, pl.idx[kT16V4], t, kT16V4);
