@@ -3,15 +3,20 @@
 
 A step is one Gefen iteration (Algorithm 1) over all 182 tensors (1,479,100,416
 fp32 parameters, bf16 gradients, u8 codes), with the workload's cadence: every
-10th step also histograms the normalised momentum (65536 cells) and refits the
-256-level codebook by the exact DP (Algorithm 3); the next step decodes with
-the old codebook and encodes with the new one.  Blocks are inferred once from
-the first gradient (Algorithm 2) and the first codebook is learned from it.
+10th step also histograms the normalised momentum (4096 cells, 16 per level)
+and refits the 256-level codebook by the exact DP (Algorithm 3); the next step
+decodes with the old codebook and encodes with the new one.  Blocks are
+inferred once from the first gradient (Algorithm 2) and the first codebook is
+learned from it.
+
+`--workload flat:N:P` runs one flat tensor of N parameters with blocks of P
+(given, not inferred): the small case the kernel profiles are taken on.
 
 Prints one JSON line.  `value` is whole-job parameters updated per second over
-the timed steps (refit steps included); `e2e` is the same metric with the
-gradient copied in from pinned host memory and the updated parameters copied
-back every step.  `--impl reference` times the CPU oracle instead, on a bounded
+the timed steps (refit steps included); `e2e` is the same metric through the
+public call with the gradient copied in from pinned host memory and the step's
+status word read back every step (and, as a second figure, all updated
+parameters copied back too).  `--impl reference` times the CPU oracle instead, on a bounded
 sample of the same workload.
 """
 from __future__ import annotations
@@ -33,7 +38,7 @@ sys.path.insert(0, ROOT)
 import numpy as np  # noqa: E402
 import torch  # noqa: E402
 
-WORKLOAD = "llama-1.5b"
+WORKLOAD = "llama-1.5b"  # the default; --workload selects another
 METRIC = "Gefen step throughput (Gparams/s)"
 UNIT = "Gparams/s"
 REFIT_EVERY = 10
@@ -164,6 +169,18 @@ def launches_per_call(periods, flags_hist: bool) -> int:
     return n + (1 if flags_hist else 0)
 
 
+def workload_specs(synth, name: str):
+    """Tensor specs of a workload, and its periods when they are given rather
+    than inferred (flat:N:P)."""
+    if name.startswith("flat:"):
+        _, n, p = name.split(":")
+        n, p = int(float(n)), int(p)
+        if n % p:
+            raise SystemExit(f"flat workload: {n} is not a multiple of {p}")
+        return synth.flat_set(n, p), [p]
+    return synth.CONFIGS[name](), None
+
+
 def period_summary(specs, periods):
     """Inferred period -> (tensors, params) over the workload."""
     out = {}
@@ -181,7 +198,7 @@ def run_gpu(args, world, rank, local):
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     G.load()
-    specs = synth.CONFIGS[WORKLOAD]()
+    specs, given_periods = workload_specs(synth, args.workload)
     offs, total = synth.pack_offsets(specs)
     nparams = synth.total_params(specs)
     stream = torch.cuda.current_stream()
@@ -192,9 +209,9 @@ def run_gpu(args, world, rank, local):
 
     # Algorithm 2 on the first gradient of every tensor
     t0 = time.perf_counter()
-    periods = []
+    periods = list(given_periods) if given_periods else []
     iws = None
-    for s, o in zip(specs, offs):
+    for s, o in zip(specs, offs) if not given_periods else []:
         need = G.gefen_infer_workspace_size(s.numel)
         if iws is None or iws.numel() < need:
             iws = G.workspace(need, dev)
@@ -341,7 +358,7 @@ def run_gpu(args, world, rank, local):
         "n_gpus": world, "steps": args.steps, "warmup": warm, "ms_per_step": elapsed_ms / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic (seeded; shapes and gradient-scale structure of the Llama-3-1.5B run)",
-        "config": {"workload": f"{WORKLOAD} shaped set: {len(specs)} tensors, {nparams} fp32 params, "
+        "config": {"workload": f"{args.workload} shaped set: {len(specs)} tensors, {nparams} fp32 params, "
                                f"{nblocks} inferred blocks; 256-level codebook; refit every {REFIT_EVERY} "
                                f"steps with {BINS} cells",
                    "params": nparams, "tensors": len(specs), "blocks": nblocks, "refit_every": REFIT_EVERY,
@@ -398,8 +415,11 @@ def refit_microbench(G, synth, dev):
 
 
 def run_e2e(G, table, theta, codes, v, sc, cb, ws, gpool, nparams, stream, args, state, one_step_ctx):
-    """Same step through the public API with host buffers: H2D of the step's
-    gradient from pinned memory, the step, D2H of the updated parameters."""
+    """Same step through the public API with host buffers: every step copies
+    its bf16 gradient in from pinned memory, runs gefen_step and reads the
+    step's result back (its 4-byte status word, gefen_step_status, which
+    waits for the step).  A second figure also copies all updated fp32
+    parameters back to pinned memory every step."""
     hist, cb_new, rws = one_step_ctx
     n = gpool[0].numel()
     g_host = torch.empty(n, dtype=torch.bfloat16, pin_memory=True)
@@ -408,50 +428,60 @@ def run_e2e(G, table, theta, codes, v, sc, cb, ws, gpool, nparams, stream, args,
     gdev = torch.empty_like(gpool[0])
     steps = max(3, min(args.steps, 10))
 
-    def e2e_step():
+    def e2e_step(readback_params: bool):
         state["t"] += 1
         gdev.copy_(g_host, non_blocking=True)
         G.gefen_step(table, theta, gdev, codes, v, sc, cb, cb, step=state["t"], workspace_buf=ws, **HP)
-        th_host.copy_(theta, non_blocking=True)
+        if readback_params:
+            th_host.copy_(theta, non_blocking=True)
+        G.gefen_step_status(ws)
 
     if state["switch"]:
         cb.copy_(cb_new)
         state["switch"] = False
-    for _ in range(2):
-        e2e_step()
-    torch.cuda.synchronize()
-    a = torch.cuda.Event(enable_timing=True)
-    b = torch.cuda.Event(enable_timing=True)
-    a.record(stream)
-    for _ in range(steps):
-        e2e_step()
-    b.record(stream)
-    torch.cuda.synchronize()
-    ms = a.elapsed_time(b)
-    return {"value": nparams * steps / (ms * 1e-3) / 1e9, "unit": UNIT, "steps": steps,
-            "h2d_bytes_per_step": 2 * n, "d2h_bytes_per_step": 4 * theta.numel()}
+    out = {}
+    for key, rb in (("status", False), ("params", True)):
+        for _ in range(2):
+            e2e_step(rb)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(steps):
+            e2e_step(rb)
+        torch.cuda.synchronize()
+        out[key] = time.perf_counter() - t0
+    return {"value": nparams * steps / out["status"] / 1e9, "unit": UNIT, "steps": steps,
+            "h2d_bytes_per_step": 2 * n, "d2h_bytes_per_step": 4,
+            "result_read": "the step's status word (gefen_step_status), every step",
+            "with_params_readback": {"value": nparams * steps / out["params"] / 1e9, "unit": UNIT,
+                                     "h2d_bytes_per_step": 2 * n, "d2h_bytes_per_step": 4 * theta.numel() + 4}}
 
 
 # ------------------------------------------------------------ CPU oracle arm
-def oracle_sample_data(max_params: int):
-    """Whole tensors of the workload (first tensors first, the 262M embedding
-    left out) up to about `max_params` parameters, with their row-length
-    periods: host arrays the oracle steps in place."""
+def oracle_sample_data(max_params: int, workload: str):
+    """Whole tensors of the workload (first tensors first, the first one, the
+    embedding, left out) up to about `max_params` parameters, with their
+    row-length periods (a flat workload: a prefix of whole blocks): host
+    arrays the oracle steps in place."""
     from paper_2606_13894_gb300 import synth
 
-    specs = synth.CONFIGS[WORKLOAD]()
+    specs, given = workload_specs(synth, workload)
+    if given:
+        pg = given[0]
+        specs = synth.flat_set(max(pg, min(specs[0].numel, max_params) // pg * pg), pg)
+    else:
+        specs = specs[1:]
     rng = np.random.default_rng(SEED)
     cb = np.concatenate([[-1.0], np.sort(np.clip(rng.standard_t(4, K - 2) * 0.1, -0.99, 0.99)),
                          [1.0]]).astype(np.float32)
     out, done = [], 0
-    for s in specs[1:]:
+    for s in specs:
         if done >= max_params:
             break
         n = s.numel
         g = synth.draw_grads([s], SEED, step=1, device="cpu")[:n]
         bits = g.view(torch.int16).numpy().view(np.uint16).copy()
         th = synth.init_params([s], SEED, device="cpu")[:n].numpy().copy()
-        p = s.cols if len(s.shape) > 1 else n
+        p = given[0] if given else (s.cols if len(s.shape) > 1 else n)
         out.append(dict(name=s.name, theta=th, bits=bits, p=p,
                         codes=np.full(n, int(np.argmin(np.abs(cb))), np.uint8),
                         v=np.zeros(n // p, np.float32), s=np.zeros(n // p, np.float32)))
@@ -469,14 +499,14 @@ def oracle_steps(data, cb, t):
 
 def cpu_baseline(args):
     import oracle
-    data, cb, done = oracle_sample_data(args.cpu_params)
+    data, cb, done = oracle_sample_data(args.cpu_params, args.workload)
     secs, t = 0.0, 0
     while secs < args.cpu_budget or t == 0:
         t += 1
         secs += oracle_steps(data, cb, t)
     return {"value": done * t / secs / 1e9, "unit": UNIT, "cores": 1, "kind": "oracle",
             "sample": f"{t} oracle steps (single thread, double precision) over {len(data)} whole tensors "
-                      f"of the {WORKLOAD} set ({done} params: {data[0]['name']} .. {data[-1]['name']}), "
+                      f"of the {args.workload} set ({done} params: {data[0]['name']} .. {data[-1]['name']}), "
                       f"{secs:.1f} s",
             "threads_available": os.cpu_count(), "oracle_threads": oracle.num_threads()}
 
@@ -485,7 +515,7 @@ def run_reference(args, world, rank):
     if rank != 0:
         return None
     warm = max(3, args.warmup)
-    data, cb, done = oracle_sample_data(int(args.ref_params))
+    data, cb, done = oracle_sample_data(int(args.ref_params), args.workload)
     t = 0
     for _ in range(warm):
         t += 1
@@ -499,10 +529,10 @@ def run_reference(args, world, rank):
             "steps": args.steps, "warmup": warm, "ms_per_step": secs * 1e3 / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic (seeded)",
-            "config": {"workload": f"{WORKLOAD} shaped set, bounded sample: {len(data)} whole tensors "
+            "config": {"workload": f"{args.workload} shaped set, bounded sample: {len(data)} whole tensors "
                                    f"({done} params) per step, oracle step"},
             "cpu_baseline": {"value": val, "unit": UNIT, "cores": 1, "kind": "oracle",
-                             "sample": f"{done} params per step ({len(data)} tensors of the {WORKLOAD} set)"},
+                             "sample": f"{done} params per step ({len(data)} tensors of the {args.workload} set)"},
             "e2e": {"value": val, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
@@ -517,6 +547,8 @@ def main():
     ap.add_argument("--ref-params", type=float, default=20e6, help="oracle params per reference step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-microbench", action="store_true", help="skip the 65536-cell refit measurement")
+    ap.add_argument("--workload", default=WORKLOAD,
+                    help="llama-1.5b (default), gpt2-125m, tiny, or flat:N:P (one tensor, blocks of P)")
     args = ap.parse_args()
     world, rank, local = dist_env()
     if args.impl == "reference":
