@@ -138,6 +138,24 @@ class Clocks:
                 "reasons": reasons, "samples": len(rows)}
 
 
+def job_time_ms(elapsed_ms: float, world: int, device) -> float:
+    """The job's time over the timed steps: the slowest rank's (every rank
+    starts after the same barrier), agreed by all ranks."""
+    if world == 1:
+        return elapsed_ms
+    import torch.distributed as dist
+    t = torch.tensor([elapsed_ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.barrier()
+    return float(t.item())
+
+
+def whole_job_value(params_per_rank: int, world: int, steps: int, job_ms: float) -> float:
+    """Parameters all replicas updated per second (each rank steps its own
+    copy of the workload: weak scaling), in Gparams/s."""
+    return world * params_per_rank * steps / (job_ms * 1e-3) / 1e9
+
+
 def dist_env():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -318,13 +336,7 @@ def run_gpu(args, world, rank, local):
     ck = clocks.stop()
     G.gefen_step_status(ws)  # raises if a bounded device wait gave up
     G.gefen_step_status(ws_b)
-    elapsed_ms = ev0.elapsed_time(ev1)
-    if world > 1:
-        import torch.distributed as dist
-        tt = torch.tensor([elapsed_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX, group=group)
-        elapsed_ms = float(tt.item())
-        dist.barrier()
+    elapsed_ms = job_time_ms(ev0.elapsed_time(ev1), world, dev)
 
     plain_ms = [a.elapsed_time(b) for a, b in step_events]
     refit_step_ms = [a.elapsed_time(b) for a, b, _ in refit_events]
@@ -354,7 +366,7 @@ def run_gpu(args, world, rank, local):
     launches = (args.steps - nref) * n_launch_plain + nref * n_launch_refit
 
     res = {
-        "metric": METRIC, "value": world * nparams * args.steps / (elapsed_ms * 1e-3) / 1e9, "unit": UNIT,
+        "metric": METRIC, "value": whole_job_value(nparams, world, args.steps, elapsed_ms), "unit": UNIT,
         "n_gpus": world, "steps": args.steps, "warmup": warm, "ms_per_step": elapsed_ms / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic (seeded; shapes and gradient-scale structure of the Llama-3-1.5B run)",
