@@ -173,7 +173,9 @@ gefen_status_t gefen_refit_codebook(const float* x, int64_t n, const uint64_t* h
 
 /* Device-side status of the last gefen_refit_codebook() that used this
  * workspace; synchronises `stream`.  k_eff_out (host, nullable) receives the
- * number of levels the DP used. */
+ * number of levels the DP used.  GEFEN_EDEVICE: the moment bound above was
+ * exceeded; GEFEN_ETIMEOUT: a bounded wait between DP levels gave up (the
+ * outputs are then undefined). */
 gefen_status_t gefen_refit_status(const void* workspace, int32_t* k_eff_out,
                                   gefen_stream_t stream);
 
@@ -195,7 +197,7 @@ gefen_status_t gefen_refit_tables(const void* workspace, int32_t bins, int32_t k
  *
  * Same inputs, outputs and results as gefen_refit_codebook(); the scratch is
  * one device array inside the library, sized for bins <= 4096 and k <= 256
- * (about 12.9 MB, held on every device that loads the library until the
+ * (about 21.2 MB, held on every device that loads the library until the
  * process exits).  Larger requests return GEFEN_EUNSUPPORTED.  It allocates
  * nothing: no cudaMalloc, cudaFree or allocating library call.
  *

@@ -17,12 +17,12 @@
 // D[.][k'-1] does not decrease along r (more cells for the same levels never
 // cost less).  So for l in [a, e]:  value(l) >= D[a-1][k'-1] + cost(e..r).
 // A 32-wide window around a hint (the previous level's split at r, moved by
-// its share of the last cell) gives the best screened value u, one candidate
-// per lane; the rest of [k', r] is searched by 32-way subdivision (one run
+// its share of the last cell; on level 2, the best of 32 evenly spaced
+// candidates) gives the best screened value u, one candidate per lane; the rest of [k', r] is searched by 32-way subdivision (one run
 // bound per lane), dropping every run whose bound exceeds u by more than 2^-34
 // relative.  Survivors (near-ties only) get the
-// canonical fp64 value; their minimum, ties to the smallest l, equals the full
-// scan bit for bit.
+// canonical fp64 value once the final bound is known; their minimum, ties to
+// the smallest l, equals the full scan bit for bit.
 #include <algorithm>
 #include <cmath>
 #include <mutex>
@@ -36,11 +36,9 @@ namespace {
 
 constexpr int kDpThreads = 64;
 constexpr float kEps = 5.820766091346741e-11f;  // 2^-34: exclusion margin (screen error < 2^-41)
-constexpr int kWin = 16;                         // window around the hint
-constexpr int kLeaf = 8;                         // runs this short are screened one by one
 
 struct Header {
-    int32_t status;  // 0 ok, 1 moment overflow (N (B-1)^2 >= 2^64)
+    int32_t status;  // 0 ok, 1 moment overflow (N (B-1)^2 >= 2^64), 2 a level barrier timed out
     int32_t b;       // nonempty cells
     int32_t k_eff;   // levels the DP uses (b <= 1: b)
     int32_t pad;
@@ -55,11 +53,12 @@ struct DpWs {
     uint64_t* P2;
     double* D;     // (k+1) x (B+1)
     int32_t* A;    // (k+1) x (B+1)
-    float2* E;     // 2 x (B+2): E[l] = (hi, lo) of D[level][l-1] for the next level
+    float2* E;     // (k+1) x (B+2): row kk, entry l = (hi, lo) of D[kk][l-1], read by level kk+1
+    uint32_t* sync;  // [0]: level-barrier arrivals; [kk]: next end position of level kk
 };
 
 struct DpLayout {
-    size_t hdr, hist, idx, P0, P1, P2, D, A, E, total;
+    size_t hdr, hist, idx, P0, P1, P2, D, A, E, sync, total;
 };
 
 // Workspace: status header at offset 0 (so it can be read without knowing the
@@ -76,7 +75,8 @@ DpLayout dp_layout(int B, int k) {
     L.P2 = o;  o += align_up(n1 * sizeof(uint64_t));
     L.D = o;   o += align_up(static_cast<size_t>(k + 1) * n1 * sizeof(double));
     L.A = o;   o += align_up(static_cast<size_t>(k + 1) * n1 * sizeof(int32_t));
-    L.E = o;   o += align_up(2 * (n1 + 1) * sizeof(float2));
+    L.E = o;   o += align_up(static_cast<size_t>(k + 1) * (n1 + 1) * sizeof(float2));
+    L.sync = o; o += align_up(static_cast<size_t>(k + 2) * sizeof(uint32_t));
     L.total = o;
     return L;
 }
@@ -93,6 +93,7 @@ DpWs dp_ws(void* base, int B, int k) {
     w.D = reinterpret_cast<double*>(p + L.D);
     w.A = reinterpret_cast<int32_t*>(p + L.A);
     w.E = reinterpret_cast<float2*>(p + L.E);
+    w.sync = reinterpret_cast<uint32_t*>(p + L.sync);
     return w;
 }
 
@@ -194,14 +195,14 @@ __device__ __forceinline__ ff cost_ff_interior(const Run& q) {
 __device__ __forceinline__ bool excluded(ff lb, ff u) {
     return ff_sub(lb, u).hi > kEps * (lb.hi + u.hi);
 }
+// Every level writes its own rows of D, A and E once, past L1, and they are
+// read only by later levels (after the grid barrier), so no SM can hold a stale
+// copy and the reads may go through L1.
 __device__ __forceinline__ ff ld_ff(const float2* E, int l) {
-    const float2 e = E[l];
+    const float2 e = __ldca(E + l);
     return ff{e.x, e.y};
 }
 
-__device__ __forceinline__ double cost64_interior(const Run& q) {
-    return __ddiv_rn(u128_to_double_rn(interior_num(q.s0, q.s1, q.s2)), __ull2double_rn(q.s0));
-}
 
 // ---------------------------------------------------------------- kernels
 // Compaction of nonempty cells and exact prefix moments (one CTA).
@@ -213,6 +214,7 @@ __global__ void __launch_bounds__(kPrefixThreads) k_dp_prefix(const uint64_t* __
     __shared__ int64_t s_p1[kPrefixThreads];
     __shared__ uint64_t s_hi[kPrefixThreads];
     const int t = threadIdx.x;
+    if (t < k + 2) W.sync[t] = 0u;
     const int per = (B + kPrefixThreads - 1) / kPrefixThreads;
     const int i0 = min(B, t * per), i1 = min(B, i0 + per);
     uint64_t cnt = 0, p0 = 0, p2 = 0, hi = 0;
@@ -303,7 +305,7 @@ __global__ void __launch_bounds__(kDpThreads) k_dp_level1(int B, DpWs W) {
         W.A[n1 + r] = (r >= 1 && r <= h.b) ? 1 : 0;
     }
     const ff e = d_to_ff(d);
-    W.E[1 * (n1 + 1) + g] = make_float2(e.hi, e.lo);  // row 1 of the rolling E buffer
+    W.E[1 * (n1 + 1) + g] = make_float2(e.hi, e.lo);  // row 1 of E
 }
 
 // Candidate screen + canonical evaluation for one (r, level) -- interior.
@@ -316,15 +318,18 @@ __device__ __forceinline__ void take(Best& b, double v, int l) {
     if (v < b.v || (v == b.v && l < b.l)) { b.v = v; b.l = l; }
 }
 
-// Lexicographic (hi, lo) minimum over the warp.
+// Lexicographic (hi, lo) minimum over the warp.  Screened values are >= 0 or
+// +inf, so hi orders like its bit pattern; lo has either sign and is mapped to
+// an order-preserving signed key.  Two integer warp reductions.
+__device__ __forceinline__ int lo_key(float x) {
+    const int b = __float_as_int(x);
+    return b >= 0 ? b : (b ^ 0x7FFFFFFF);
+}
 __device__ __forceinline__ ff warp_min_ff(ff v) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        const float oh = __shfl_xor_sync(0xffffffffu, v.hi, o);
-        const float ol = __shfl_xor_sync(0xffffffffu, v.lo, o);
-        if (oh < v.hi || (oh == v.hi && ol < v.lo)) v = ff{oh, ol};
-    }
-    return v;
+    const unsigned hb = __float_as_uint(v.hi);
+    const unsigned hm = __reduce_min_sync(0xffffffffu, hb);
+    const int lk = __reduce_min_sync(0xffffffffu, hb == hm ? lo_key(v.lo) : 0x7FFFFFFF);
+    return ff{__uint_as_float(hm), __int_as_float(lk >= 0 ? lk : (lk ^ 0x7FFFFFFF))};
 }
 __device__ __forceinline__ Best warp_min_best(Best b) {
 #pragma unroll
@@ -336,7 +341,7 @@ __device__ __forceinline__ Best warp_min_best(Best b) {
     return b;
 }
 
-constexpr int kDpWarps = 8;      // warps (end positions) per CTA
+constexpr int kDpWarps = 16;     // warps (end positions at a time) per CTA
 constexpr int kStackCap = 192;   // runs pending per warp
 
 // Everything one warp needs to screen and evaluate candidates for one r.
@@ -355,30 +360,69 @@ __device__ __forceinline__ ff run_cost_ff(const RowCtx& c, int l) {
     const Run q = run_of(*c.W, l, c.P0r, c.P1r, c.P2r);
     return c.last ? u128_to_ff(fixed_num(q.s0, q.s1, q.s2, c.B, -1)) : cost_ff_interior(q);
 }
-__device__ __forceinline__ double run_cost_64(const RowCtx& c, int l) {
+
+// Canonical value of candidate l: D[l-1] + cost(l..r), each rounded as the
+// oracle rounds them (fp64; slow on this part, so used only for near-ties).
+__device__ __forceinline__ double canonical(const RowCtx& c, int l) {
     const Run q = run_of(*c.W, l, c.P0r, c.P1r, c.P2r);
-    return c.last ? u128_to_double_rn(fixed_num(q.s0, q.s1, q.s2, c.B, -1)) : cost64_interior(q);
+    const double dprev = __ldca(c.Dp + l - 1);
+    const double cost = c.last ? u128_to_double_rn(fixed_num(q.s0, q.s1, q.s2, c.B, -1))
+                               : __ddiv_rn(u128_to_double_rn(interior_num(q.s0, q.s1, q.s2)), __ull2double_rn(q.s0));
+    return __dadd_rn(dprev, cost);
 }
 
-// One round over up to 32 consecutive candidates [a, a+31] ∩ [a, e].
-__device__ __forceinline__ void eval_candidates(const RowCtx& c, int a, int e, int lane, ff& u, Best& bst) {
-    const int l = a + lane;
+// Search state of one warp: u is the best screened value seen; each lane
+// keeps at most one pending candidate (one not excluded when it was screened),
+// whose canonical value is taken only if the final u still does not exclude
+// it.  A second pending candidate in the same lane first settles the first.
+// Every candidate the final u does not exclude thus gets its canonical value,
+// and the best of those is the full scan's.
+struct Search {
+    ff u;
+    int pl;  // pending candidate of this lane, 0 if none
+    ff pv;   // its screened value
+    Best bst;
+};
+
+__device__ __forceinline__ void settle(const RowCtx& c, Search& S) {
+    if (S.pl != 0 && !excluded(S.pv, S.u)) take(S.bst, canonical(c, S.pl), S.pl);
+    S.pl = 0;
+}
+
+// One round over up to 32 candidates a, a+st, ..., one per lane, up to e.
+__device__ __forceinline__ void eval_candidates(const RowCtx& c, int a, int e, int lane, Search& S, int st = 1) {
+    const int l = a + lane * st;
     const bool in = l <= e;
     ff v{INFINITY, 0.0f};
     if (in) v = ff_add(ld_ff(c.Ep, l), run_cost_ff(c, l));
     const ff vm = warp_min_ff(v);
-    if (vm.hi < u.hi || (vm.hi == u.hi && vm.lo < u.lo)) u = vm;
-    if (in && !excluded(v, u)) take(bst, __dadd_rn(c.Dp[l - 1], run_cost_64(c, l)), l);
+    if (vm.hi < S.u.hi || (vm.hi == S.u.hi && vm.lo < S.u.lo)) S.u = vm;
+    if (in && !excluded(v, S.u)) {
+        settle(c, S);
+        S.pl = l;
+        S.pv = v;
+    }
 }
 
 __device__ Best search_row(const RowCtx& c, int kk, int hint, int lane, int2* stack) {
-    Best bst{INFINITY, 0};
-    ff u{INFINITY, 0.0f};
+    Search S;
+    S.u = ff{INFINITY, 0.0f};
+    S.pl = 0;
+    S.pv = ff{INFINITY, 0.0f};
+    S.bst = Best{INFINITY, 0};
     const int r = c.r;
+    if (kk == 2 && r - kk >= 64) {
+        // level 2: the previous level's split (always 1) says nothing, so
+        // sample 32 evenly spaced candidates and centre the window on the best
+        const int st = (r - kk) / 31;
+        eval_candidates(c, kk, r, lane, S, st);
+        const unsigned at = __ballot_sync(0xffffffffu, S.pl != 0 && S.pv.hi == S.u.hi && S.pv.lo == S.u.lo);
+        hint = at ? __shfl_sync(0xffffffffu, S.pl, __ffs(at) - 1) : kk + (r - kk) / 2;
+    }
     int w0 = max(kk, hint - 8);
     const int w1 = min(r, w0 + 31);
     w0 = max(kk, w1 - 31);
-    eval_candidates(c, w0, w1, lane, u, bst);
+    eval_candidates(c, w0, w1, lane, S);
     int sp = 0;  // warp-uniform
     if (lane == 0) {
         if (w1 < r) stack[sp] = make_int2(w1 + 1, r);
@@ -391,19 +435,19 @@ __device__ Best search_row(const RowCtx& c, int kk, int hint, int lane, int2* st
         __syncwarp();
         const int a = run.x, e = run.y, width = e - a + 1;
         if (width <= 32) {
-            eval_candidates(c, a, e, lane, u, bst);
+            eval_candidates(c, a, e, lane, S);
             continue;
         }
         // 32 sub-runs; lane i bounds [ca, ce] by D[ca-1] + cost(ce..r)
         const int cw = (width + 31) >> 5;
         const int ca = a + lane * cw, ce = min(e, ca + cw - 1);
         bool keep = false;
-        if (ca <= e) keep = !excluded(ff_add(ld_ff(c.Ep, ca), run_cost_ff(c, ce)), u);
+        if (ca <= e) keep = !excluded(ff_add(ld_ff(c.Ep, ca), run_cost_ff(c, ce)), S.u);
         const unsigned mask = __ballot_sync(0xffffffffu, keep);
         const int cnt = __popc(mask);
         if (sp + cnt > kStackCap) {
             // no room to split: screen the run directly (never expected)
-            for (int b = a; b <= e; b += 32) eval_candidates(c, b, min(e, b + 31), lane, u, bst);
+            for (int b = a; b <= e; b += 32) eval_candidates(c, b, min(e, b + 31), lane, S);
             continue;
         }
         // nearest the window on top: left of the window -> highest sub-run last
@@ -413,19 +457,15 @@ __device__ Best search_row(const RowCtx& c, int kk, int hint, int lane, int2* st
         sp += cnt;
         __syncwarp();
     }
-    return warp_min_best(bst);
+    settle(c, S);
+    return warp_min_best(S.bst);
 }
 
-// Level kk: interior (2 <= kk < k_eff) for every r, or the last level
-// (kk == k_eff) for r = b only, or nothing defined (kk > k_eff).  One warp per
-// r in [0, B]; every D[kk][r] is written (+inf where undefined).
-__global__ void __launch_bounds__(kDpWarps * 32) k_dp_level(int B, int kk, DpWs W) {
-    __shared__ int2 s_stack[kDpWarps][kStackCap];
-    const Header h = *W.hdr;
-    if (h.status) return;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int r = blockIdx.x * kDpWarps + warp;
-    if (r > B) return;
+// Level kk at end position r: interior (2 <= kk < k_eff) for every r, or the
+// last level (kk == k_eff) for r = b only, or nothing defined (kk > k_eff).
+// Every D[kk][r] is written (+inf where undefined).
+__device__ __forceinline__ void level_row(int B, int kk, int r, const DpWs& W, const Header& h, int lane,
+                                          int2* stack) {
     const int n1 = B + 1;
     const bool last = (kk == h.k_eff);
     const bool active = kk <= h.k_eff && r <= h.b && (last ? (r == h.b) : (r >= kk));
@@ -435,7 +475,7 @@ __global__ void __launch_bounds__(kDpWarps * 32) k_dp_level(int B, int kk, DpWs 
         RowCtx c;
         c.W = &W;
         c.Dp = W.D + static_cast<size_t>(kk - 1) * n1;
-        c.Ep = W.E + static_cast<size_t>((kk - 1) & 1) * (n1 + 1);
+        c.Ep = W.E + static_cast<size_t>(kk - 1) * (n1 + 1);
         c.P0r = W.P0[r];
         c.P1r = W.P1[r];
         c.P2r = W.P2[r];
@@ -443,19 +483,70 @@ __global__ void __launch_bounds__(kDpWarps * 32) k_dp_level(int B, int kk, DpWs 
         c.r = r;
         c.last = last;
         // hint: the previous level's split at r, moved by its share of the last cell
-        const int hp = max(kk, W.A[static_cast<size_t>(kk - 1) * n1 + r]);
+        const int hp = max(kk, __ldca(W.A + static_cast<size_t>(kk - 1) * n1 + r));
         const int hint = hp + (r - hp) / kk;
-        const Best b = search_row(c, kk, hint, lane, s_stack[warp]);
+        const Best b = search_row(c, kk, hint, lane, stack);
         d = b.v;
         al = b.l;
     }
     if (lane == 0) {
-        W.D[static_cast<size_t>(kk) * n1 + r] = d;
-        W.A[static_cast<size_t>(kk) * n1 + r] = al;
+        // stored past L1 (.cg): no SM may cache part of a row before the level ends
+        __stcg(W.D + static_cast<size_t>(kk) * n1 + r, d);
+        __stcg(W.A + static_cast<size_t>(kk) * n1 + r, al);
         const ff e = d_to_ff(d);
-        float2* En = W.E + static_cast<size_t>(kk & 1) * (n1 + 1);
-        En[r + 1] = make_float2(e.hi, e.lo);
-        if (r == 0) En[0] = make_float2(INFINITY, 0.0f);
+        float2* En = W.E + static_cast<size_t>(kk) * (n1 + 1);
+        __stcg(En + r + 1, make_float2(e.hi, e.lo));
+        if (r == 0) __stcg(En, make_float2(INFINITY, 0.0f));
+    }
+}
+
+__device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+// Levels 2..k in one cooperative launch (every CTA resident).  Warp w of the
+// grid takes end position w of each level, and positions past the grid's
+// warps come from a counter; a grid barrier separates the levels.  The
+// barrier's wait gives up after about a second (status 2), so a lost CTA
+// cannot hang the GPU.
+__global__ void __launch_bounds__(kDpWarps * 32) k_dp_levels(int B, int k, DpWs W) {
+    __shared__ int2 s_stack[kDpWarps][kStackCap];
+    __shared__ int s_abort;
+    const Header h = *W.hdr;
+    if (h.status) return;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t G = gridDim.x;
+    const int nwarps = static_cast<int>(G) * kDpWarps;
+    for (int kk = 2; kk <= k; ++kk) {
+        int r = static_cast<int>(blockIdx.x) * kDpWarps + warp;
+        while (r <= B) {
+            level_row(B, kk, r, W, h, lane, s_stack[warp]);
+            if (nwarps > B) break;  // every position had a warp of its own
+            int nr = 0;
+            if (lane == 0) nr = nwarps + static_cast<int>(atomicAdd(W.sync + kk, 1u));
+            r = __shfl_sync(0xffffffffu, nr, 0);
+        }
+        if (kk == k) break;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            __threadfence();  // this CTA's rows of level kk before its arrival
+            atomicAdd(W.sync, 1u);
+            const uint32_t target = static_cast<uint32_t>(kk - 1) * G;
+            const long long t0 = clock64();
+            int ab = 0;
+            while (ld_acquire(W.sync) < target) {
+                if (clock64() - t0 > (1ll << 31)) {
+                    ab = 1;
+                    atomicExch(&W.hdr->status, 2);
+                    break;
+                }
+            }
+            s_abort = ab;
+        }
+        __syncthreads();
+        if (s_abort) return;
     }
 }
 
@@ -550,8 +641,20 @@ extern "C" gefen_status_t gefen_refit_codebook(const float* x, int64_t n, const 
     k_dp_prefix<<<1, kPrefixThreads, 0, st>>>(h, bins, k, W);
     const int grid1 = (bins + 2 + kDpThreads - 1) / kDpThreads;
     k_dp_level1<<<grid1, kDpThreads, 0, st>>>(bins, W);
-    const int grid = (bins + 1 + kDpWarps - 1) / kDpWarps;
-    for (int kk = 2; kk <= k; ++kk) k_dp_level<<<grid, kDpWarps * 32, 0, st>>>(bins, kk, W);
+    {
+        static int per_sm = 0;  // resident CTAs per SM (a property of the kernel)
+        if (per_sm == 0 &&
+            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_dp_levels, kDpWarps * 32, 0) != cudaSuccess)
+            return GEFEN_ECUDA;
+        const int rows = (bins + 1 + kDpWarps - 1) / kDpWarps;  // CTAs with a row each
+        int grid = std::max(1, std::min(per_sm * device_sm_count(), rows));
+        int bb = bins, kv = k;
+        DpWs w = W;
+        void* args[] = {&bb, &kv, &w};
+        if (cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(k_dp_levels), dim3(grid), dim3(kDpWarps * 32),
+                                        args, 0, st) != cudaSuccess)
+            return GEFEN_ECUDA;
+    }
     k_dp_backtrack<<<1, 32, 0, st>>>(bins, k, W, codebook_out, cell_start_out, cost_out);
     if (cudaGetLastError() != cudaSuccess) return GEFEN_ECUDA;
     return GEFEN_OK;
@@ -564,6 +667,7 @@ extern "C" gefen_status_t gefen_refit_status(const void* workspace, int32_t* k_e
     if (cudaMemcpyAsync(&h, workspace, sizeof(h), cudaMemcpyDeviceToHost, st) != cudaSuccess) return GEFEN_ECUDA;
     if (cudaStreamSynchronize(st) != cudaSuccess) return GEFEN_ECUDA;
     if (k_eff_out) *k_eff_out = h.k_eff;
+    if (h.status == 2) return GEFEN_ETIMEOUT;
     return h.status ? GEFEN_EDEVICE : GEFEN_OK;
 }
 
@@ -601,7 +705,8 @@ constexpr size_t kStaticScratchBytes =
     cx_align(size_t(kStaticMaxBins + 1) * sizeof(int32_t)) + 3 * cx_align(size_t(kStaticMaxBins + 1) * 8) +
     cx_align(size_t(kStaticMaxLevels + 1) * (kStaticMaxBins + 1) * sizeof(double)) +
     cx_align(size_t(kStaticMaxLevels + 1) * (kStaticMaxBins + 1) * sizeof(int32_t)) +
-    cx_align(2 * size_t(kStaticMaxBins + 2) * sizeof(float2));
+    cx_align(size_t(kStaticMaxLevels + 1) * (kStaticMaxBins + 2) * sizeof(float2)) +
+    cx_align(size_t(kStaticMaxLevels + 2) * sizeof(uint32_t));
 
 __device__ __align__(256) unsigned char g_refit_scratch[kStaticScratchBytes];
 
