@@ -87,7 +87,9 @@ struct Ptrs {
     const float* cb_dec;
     const float* cb_enc;
     int k;
-    float* xstage;      // histogram input staging (HIST modes)
+    float* xstage;      // histogram input staging (HIST modes, kernels that do not count in place)
+    uint64_t* hist;     // the histogram (HIST modes)
+    int bins;
     double* part_g2;    // big path: per-chunk sum of g^2
     float* part_mx;     // big path: per-chunk max
     float4* blk_state;  // big path: per big block (s_old, s_new, fac, -)
@@ -417,9 +419,11 @@ struct StageLayout {
     static constexpr int kBytes = kC + TILE;
 };
 
-template <int TILE, int THREADS, int STAGES, int LUTR, int DECR, bool THS>
+template <int TILE, int THREADS, int STAGES, int LUTR, int DECR, bool THS, int HB>
 struct alignas(128) StreamSmem {
+    static constexpr int kHistCells = HB;  // cells counted in shared memory (0: x is staged instead)
     unsigned char stage[STAGES][StageLayout<TILE, THS>::kBytes];
+    uint32_t hist[HB > 0 ? HB : 1];
     StreamTables<LUTR, DECR> tab;
     float2 part[THREADS / 32];  // per warp: (sum g^2, max |m|)
     float2 blk[TILE / 16];      // per block, irregular shapes: (step factor, 1/s')  [grad-only: (-, absmax)]
@@ -755,7 +759,7 @@ __device__ __forceinline__ void stream_tile(Smem& sm, const Ptrs& P, const HP& h
     // straight from registers.  A zero block (inv = 0) encodes x = 0, the
     // level nearest 0, and stages NaN for the histogram.
     uint8_t* cdp = P.codes + ti.e0 + eb;
-    float* xsp = (MODE != kPlain) ? P.xstage + ti.e0 + eb : nullptr;
+    float* xsp = (MODE != kPlain && Smem::kHistCells == 0) ? P.xstage + ti.e0 + eb : nullptr;
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
         if (!live[j]) continue;
@@ -779,7 +783,18 @@ __device__ __forceinline__ void stream_tile(Smem& sm, const Ptrs& P, const HP& h
                 for (int i = 0; i < 4; ++i) x[i] = inv[j] > 0.0f ? x[i] : __int_as_float(0x7fffffff);
             }
         }
-        if (MODE != kPlain) __stcs(reinterpret_cast<float4*>(xsp + 128 * j), make_float4(x[0], x[1], x[2], x[3]));
+        if (MODE != kPlain) {
+            if (Smem::kHistCells > 0) {
+                // count x of nonzero blocks in the CTA's cells (NaN skipped)
+                if (inv[j] > 0.0f) {
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                        if (!isnan(x[i])) atomicAdd(&sm.hist[hist_cell(x[i], 0.5f * P.bins, P.bins)], 1u);
+                }
+            } else {
+                __stcs(reinterpret_cast<float4*>(xsp + 128 * j), make_float4(x[0], x[1], x[2], x[3]));
+            }
+        }
     }
 }
 
@@ -833,9 +848,9 @@ __device__ __forceinline__ void stream_loop(Smem& sm, const Launch& L, const Ptr
     }
 }
 
-template <int TILE, int THREADS, int STAGES, int LUTR, int DECR, bool THS, int MODE, int MINB>
+template <int TILE, int THREADS, int STAGES, int LUTR, int DECR, bool THS, int HB, int MODE, int MINB>
 __global__ void __launch_bounds__(THREADS, MINB) k_step_stream(const __grid_constant__ Launch L, const Ptrs P, int* err) {
-    using Smem = StreamSmem<TILE, THREADS, STAGES, LUTR, DECR, THS>;
+    using Smem = StreamSmem<TILE, THREADS, STAGES, LUTR, DECR, THS, HB>;
     static_assert(TILE == 16 * THREADS && THREADS % 32 == 0 && STAGES >= 2, "tile shape");
     static_assert(32 % LUTR == 0 && 32 % DECR == 0, "table copies");
     extern __shared__ __align__(128) unsigned char smem_raw[];
@@ -851,12 +866,22 @@ __global__ void __launch_bounds__(THREADS, MINB) k_step_stream(const __grid_cons
             if (u < L.nunits) issue_tile<TILE, MODE, THS>(sm, s, tile_info(L, u, seg), P);
         }
     }
+    if (HB > 0)
+        for (int i = threadIdx.x; i < HB; i += THREADS) sm.hist[i] = 0u;
     const int bad = build_tables<THREADS>(P, sm.tab, MODE == kGradOnly);
     const bool lut_ok = !__syncthreads_or(bad);
     if (MODE != kGradOnly && lut_ok)
         stream_loop<TILE, THREADS, STAGES, LUTR, DECR, MODE, THS, true>(sm, L, P, err, seg);
     else
         stream_loop<TILE, THREADS, STAGES, LUTR, DECR, MODE, THS, false>(sm, L, P, err, seg);
+    if (HB > 0) {
+        // add the CTA's counts to the histogram
+        __syncthreads();
+        for (int c = threadIdx.x; c < P.bins; c += THREADS) {
+            const uint32_t n = sm.hist[c];
+            if (n) atomicAdd(reinterpret_cast<unsigned long long*>(P.hist) + c, static_cast<unsigned long long>(n));
+        }
+    }
 }
 
 // ------------------------------------------- generic p <= 2048 (scalar)
@@ -1184,6 +1209,11 @@ struct StreamCfg {
 // (theta staged too), cell records in 8 copies and the decode table in 32.
 using S4KCfg = StreamCfg<4096, 256, 3, 8, 8, false, 2>;
 using S8KCfg = StreamCfg<8192, 512, 2, 8, 32, true, 1>;
+// Steps that also histogram x (refit steps) count up to kFusedBins cells in
+// shared memory; the tables give up copies to make room.
+constexpr int kFusedBins = 4096;
+using S4KHistCfg = StreamCfg<4096, 256, 3, 2, 4, false, 2>;
+using S8KHistCfg = StreamCfg<8192, 512, 2, 2, 4, true, 1>;
 constexpr int kS4KTile = S4KCfg::TILE, kS8KTile = S8KCfg::TILE;
 
 PathClass classify(int64_t p) {
@@ -1313,11 +1343,11 @@ cudaError_t launch_class(K kernel, Launch& L, const std::vector<int>& ids, const
     return cudaSuccess;
 }
 
-template <typename C, int MODE>
+template <typename C, int MODE, int HB>
 cudaError_t launch_stream(Launch& L, const std::vector<int>& ids, const gefen_tensor_t* t, PathClass c,
                           const Ptrs& P, int* err, cudaStream_t st) {
-    auto kern = k_step_stream<C::TILE, C::THREADS, C::STAGES, C::LUTR, C::DECR, C::THS, MODE, C::MINB>;
-    const int smem = static_cast<int>(sizeof(StreamSmem<C::TILE, C::THREADS, C::STAGES, C::LUTR, C::DECR, C::THS>));
+    auto kern = k_step_stream<C::TILE, C::THREADS, C::STAGES, C::LUTR, C::DECR, C::THS, HB, MODE, C::MINB>;
+    const int smem = static_cast<int>(sizeof(StreamSmem<C::TILE, C::THREADS, C::STAGES, C::LUTR, C::DECR, C::THS, HB>));
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
@@ -1333,15 +1363,24 @@ cudaError_t launch_stream(Launch& L, const std::vector<int>& ids, const gefen_te
         L, ids, t, c, C::TILE);
 }
 
+// fused: the streamed kernels count the histogram in shared memory (the
+// other kernels stage x for launch_histogram).
 template <int MODE>
-cudaError_t run_step(const Plan& pl, const gefen_tensor_t* t, Launch& L, const Ptrs& P, int* err, cudaStream_t st) {
+cudaError_t run_step(const Plan& pl, const gefen_tensor_t* t, Launch& L, const Ptrs& P, int* err, cudaStream_t st,
+                     bool fused) {
     cudaError_t e;
     e = launch_class([&](Launch& LL, int64_t u) { k_step_p1<MODE><<<dim3(u), kThreads, 0, st>>>(LL, P); },
                      L, pl.idx[kP1], t, kP1);
     if (e != cudaSuccess) return e;
-    e = launch_stream<S4KCfg, MODE>(L, pl.idx[kS4K], t, kS4K, P, err, st);
+    if (MODE != kPlain && fused)
+        e = launch_stream<S4KHistCfg, MODE, kFusedBins>(L, pl.idx[kS4K], t, kS4K, P, err, st);
+    else
+        e = launch_stream<S4KCfg, MODE, 0>(L, pl.idx[kS4K], t, kS4K, P, err, st);
     if (e != cudaSuccess) return e;
-    e = launch_stream<S8KCfg, MODE>(L, pl.idx[kS8K], t, kS8K, P, err, st);
+    if (MODE != kPlain && fused)
+        e = launch_stream<S8KHistCfg, MODE, kFusedBins>(L, pl.idx[kS8K], t, kS8K, P, err, st);
+    else
+        e = launch_stream<S8KCfg, MODE, 0>(L, pl.idx[kS8K], t, kS8K, P, err, st);
     if (e != cudaSuccess) return e;
     e = launch_class([&](Launch& LL, int64_t u) { k_step_tile16<4, MODE><<<dim3(u), kThreads, 0, st>>>(LL, P); },
                      L, pl.idx[kT16V4], t, kT16V4);
@@ -1429,6 +1468,8 @@ extern "C" gefen_status_t gefen_step(const gefen_tensor_t* tensors, int32_t nten
     P.cb_enc = codebook_enc;
     P.k = grad_only ? 2 : k;
     P.xstage = want_hist ? reinterpret_cast<float*>(ws + wl.xstage) : nullptr;
+    P.hist = hist;
+    P.bins = hist_bins;
     P.part_g2 = reinterpret_cast<double*>(ws + wl.part_g2);
     P.part_mx = reinterpret_cast<float*>(ws + wl.part_mx);
     P.blk_state = reinterpret_cast<float4*>(ws + wl.blk_state);
@@ -1450,14 +1491,19 @@ extern "C" gefen_status_t gefen_step(const gefen_tensor_t* tensors, int32_t nten
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     cudaError_t e;
     int* err = reinterpret_cast<int*>(ws + wl.header);
-    if (grad_only) e = run_step<kGradOnly>(pl, tensors, L, P, err, st);
-    else if (flags & GEFEN_HIST) e = run_step<kHist>(pl, tensors, L, P, err, st);
-    else e = run_step<kPlain>(pl, tensors, L, P, err, st);
+    const bool fused = want_hist && hist_bins <= kFusedBins;
+    if (grad_only) e = run_step<kGradOnly>(pl, tensors, L, P, err, st, fused);
+    else if (flags & GEFEN_HIST) e = run_step<kHist>(pl, tensors, L, P, err, st, fused);
+    else e = run_step<kPlain>(pl, tensors, L, P, err, st, false);
     if (e != cudaSuccess) return GEFEN_ECUDA;
     if (want_hist) {
         std::vector<HistRange> rr;
-        for (int i = 0; i < ntensors; ++i)
-            if (tensors[i].numel > 0) rr.push_back({tensors[i].offset, tensors[i].numel});
+        for (int i = 0; i < ntensors; ++i) {
+            if (tensors[i].numel == 0) continue;
+            const PathClass c = classify(tensors[i].period);
+            if (fused && (c == kS4K || c == kS8K)) continue;  // counted in place
+            rr.push_back({tensors[i].offset, tensors[i].numel});
+        }
         if (!rr.empty() && launch_histogram(P.xstage, rr.data(), static_cast<int>(rr.size()), hist_bins, hist, st) !=
                                cudaSuccess)
             return GEFEN_ECUDA;
