@@ -1,0 +1,241 @@
+"""A torch.optim-compatible Gefen optimizer (AdamW's signature) on libgefen.
+
+Each parameter group's parameters are moved into one flat fp32 arena on first
+use (the parameters become views of it, so the model sees every update); their
+gradients are gathered into a bf16 arena before each step.  The first step
+infers every tensor's blocks from its gradient (Algorithm 2, unless periods
+are given) and learns the first codebook from that gradient (Algorithm 3 on
+the histogram of g / block absmax); from then on each step is one gefen_step
+call over the whole group (Algorithm 1).  With refit_every = N > 0, every N-th
+step also histograms the normalised momentum and refits the codebook; the next
+step decodes with the old codebook and encodes with the new one.
+
+All arithmetic of the step runs in the library's CUDA kernels; this module
+only lays out memory and sequences calls.  CUDA fp32 parameters are required:
+there is no CPU path.
+"""
+from __future__ import annotations
+
+from typing import Dict, List, Optional, Sequence
+
+import torch
+
+from . import gefen as G
+
+ALIGN = 64  # elements between tensors in an arena (16 is the library's minimum)
+
+
+class _Arena:
+    """The packed state of one parameter group."""
+
+    def __init__(self, params: List[torch.nn.Parameter], levels: int, bins: int):
+        dev = params[0].device
+        self.params = params
+        self.offsets, o = [], 0
+        for p in params:
+            self.offsets.append(o)
+            o += (p.numel() + ALIGN - 1) // ALIGN * ALIGN
+        self.total = max(o, ALIGN)
+        self.theta = torch.zeros(self.total, dtype=torch.float32, device=dev)
+        with torch.no_grad():
+            for p, off in zip(params, self.offsets):
+                self.theta[off:off + p.numel()].copy_(p.detach().reshape(-1))
+                p.data = self.theta[off:off + p.numel()].view_as(p)
+        self.grads = torch.zeros(self.total, dtype=torch.bfloat16, device=dev)
+        self.gviews = [self.grads[off:off + p.numel()].view_as(p) for p, off in zip(params, self.offsets)]
+        self.codes = torch.zeros(self.total, dtype=torch.uint8, device=dev)
+        self.levels, self.bins = levels, bins
+        self.cb = torch.empty(levels, dtype=torch.float32, device=dev)
+        self.cb_new = torch.empty(levels, dtype=torch.float32, device=dev)
+        self.hist = torch.zeros(bins, dtype=torch.int64, device=dev)
+        self.periods: Optional[List[int]] = None
+        self.v = self.s = None
+        self.table = None
+        self.entries: List[tuple] = []
+        self.t = 0
+        self.switch = False  # the next step encodes with cb_new
+        self.ws = self.rws = None
+        self._sub = {}
+
+    def set_periods(self, periods: Sequence[int]):
+        self.periods = [int(p) for p in periods]
+        self.entries, b = [], 0
+        for p, off, per in zip(self.params, self.offsets, self.periods):
+            if per < 1 or p.numel() % per:
+                raise ValueError(f"period {per} does not divide a tensor of {p.numel()} elements")
+            self.entries.append((off, p.numel(), per, b))
+            b += p.numel() // per
+        dev = self.theta.device
+        self.v = torch.zeros(max(b, 1), dtype=torch.float32, device=dev)
+        self.s = torch.zeros(max(b, 1), dtype=torch.float32, device=dev)
+        self.table = G.tensor_table(self.entries)
+        self._sub = {}
+
+    def table_for(self, present: Sequence[bool]):
+        """The tensor table of the parameters that have a gradient this step."""
+        if all(present):
+            return self.table
+        key = tuple(present)
+        if key not in self._sub:
+            self._sub[key] = G.tensor_table([e for e, ok in zip(self.entries, present) if ok])
+        return self._sub[key]
+
+
+class Gefen(torch.optim.Optimizer):
+    """Gefen (Algorithm 1) with AdamW's arguments.
+
+    levels: codebook size k (256: 8-bit codes).  bins: histogram cells of the
+    codebook refit (default 16 per level).  refit_every: refit the codebook
+    every N steps (0: learn it once, from the first gradient).  periods:
+    optional block size of every parameter, all groups in order (default:
+    inferred from the first gradient, Algorithm 2).
+    Parameters without a gradient at a step are left untouched, as in AdamW.
+    """
+
+    def __init__(self, params, lr: float = 1e-3, betas=(0.9, 0.999), eps: float = 1e-8,
+                 weight_decay: float = 1e-2, *, levels: int = 256, bins: Optional[int] = None,
+                 refit_every: int = 0, periods: Optional[Sequence[int]] = None):
+        if not 0.0 <= lr or not 0.0 <= eps or not 0.0 <= weight_decay:
+            raise ValueError("lr, eps and weight_decay must be non-negative")
+        if not (0.0 <= betas[0] < 1.0 and 0.0 <= betas[1] < 1.0):
+            raise ValueError("betas must lie in [0, 1)")
+        if not 2 <= levels <= G.GEFEN_MAX_LEVELS:
+            raise ValueError(f"levels must lie in [2, {G.GEFEN_MAX_LEVELS}]")
+        defaults = dict(lr=lr, betas=tuple(betas), eps=eps, weight_decay=weight_decay)
+        super().__init__(params, defaults)
+        self.levels = int(levels)
+        self.bins = int(bins) if bins else 16 * self.levels
+        if not self.levels <= self.bins <= G.GEFEN_MAX_BINS:
+            raise ValueError(f"bins must lie in [levels, {G.GEFEN_MAX_BINS}]")
+        self.refit_every = int(refit_every)
+        self._given_periods = list(periods) if periods is not None else None
+        for group in self.param_groups:
+            for p in group["params"]:
+                if not p.is_cuda or p.dtype != torch.float32:
+                    raise ValueError("Gefen needs CUDA fp32 parameters (the library has no CPU path)")
+        G.load()  # fails loudly when the CUDA library is missing
+        self._arenas: List[Optional[_Arena]] = [None] * len(self.param_groups)
+        self._pending: Optional[list] = None
+
+    # ------------------------------------------------------------ set-up
+    def _first_step(self, gi: int, group, present):
+        params = list(group["params"])
+        A = _Arena(params, self.levels, self.bins)
+        self._arenas[gi] = A
+        if self._pending is not None and self._pending[gi] is not None:
+            self._restore(A, self._pending[gi])
+            return
+        if not all(present):
+            raise RuntimeError("the first step needs a gradient for every parameter (it infers their blocks)")
+        self._gather(A, present)
+        beta1, beta2 = group["betas"]
+        if self._given_periods is not None:
+            # the periods list follows the parameters of all groups in order
+            start = sum(len(g["params"]) for g in self.param_groups[:gi])
+            periods = self._given_periods[start:start + len(params)]
+        else:
+            periods, iws = [], None
+            for p, gv in zip(params, A.gviews):
+                need = G.gefen_infer_workspace_size(p.numel())
+                if iws is None or iws.numel() < need:
+                    iws = G.workspace(need, p.device)
+                per, _ = G.gefen_infer_blocks(gv.reshape(-1), group["eps"], workspace_buf=iws, want_scores=False)
+                periods.append(per)
+        A.set_periods(periods)
+        # first codebook: histogram of g / block absmax, then the exact DP
+        A.ws = G.gefen_step(A.table, A.theta, A.grads, A.codes, A.v, A.s, A.cb, A.cb, lr=group["lr"],
+                            beta1=beta1, beta2=beta2, eps=group["eps"], weight_decay=group["weight_decay"],
+                            step=1, flags=G.GEFEN_HIST_GRAD_ONLY, hist=A.hist, workspace_buf=A.ws)
+        A.rws = G.gefen_refit_codebook(bins=self.bins, k=self.levels, codebook_out=A.cb, hist_in=A.hist,
+                                       workspace_buf=A.rws)
+        A.codes.fill_(int(torch.argmin(A.cb.abs()).item()))  # the level nearest 0, lower index on ties
+
+    def _gather(self, A: _Arena, present):
+        src = [p.grad for p, ok in zip(A.params, present) if ok]
+        dst = [g for g, ok in zip(A.gviews, present) if ok]
+        if any(g.is_sparse for g in src):
+            raise RuntimeError("Gefen does not take sparse gradients")
+        torch._foreach_copy_(dst, src)
+
+    # --------------------------------------------------------------- step
+    @torch.no_grad()
+    def step(self, closure=None):
+        loss = None
+        if closure is not None:
+            with torch.enable_grad():
+                loss = closure()
+        for gi, group in enumerate(self.param_groups):
+            present = [p.grad is not None for p in group["params"]]
+            if not any(present):
+                continue
+            if self._arenas[gi] is None:
+                self._first_step(gi, group, present)
+            A = self._arenas[gi]
+            self._gather(A, present)
+            A.t += 1
+            beta1, beta2 = group["betas"]
+            refit = self.refit_every > 0 and A.t % self.refit_every == 0
+            enc = A.cb_new if A.switch else A.cb
+            if refit:
+                A.hist.zero_()
+            A.ws = G.gefen_step(A.table_for(present), A.theta, A.grads, A.codes, A.v, A.s, A.cb, enc,
+                                lr=group["lr"], beta1=beta1, beta2=beta2, eps=group["eps"],
+                                weight_decay=group["weight_decay"], step=A.t,
+                                flags=G.GEFEN_HIST if refit else 0, hist=A.hist if refit else None,
+                                workspace_buf=A.ws)
+            if A.switch:
+                A.cb.copy_(A.cb_new)
+                A.switch = False
+            if refit:
+                A.rws = G.gefen_refit_codebook(bins=self.bins, k=self.levels, codebook_out=A.cb_new,
+                                               hist_in=A.hist, workspace_buf=A.rws)
+                A.switch = True
+        return loss
+
+    def check(self):
+        """Waits for the device and raises if a step or refit gave up a
+        bounded wait (GEFEN_ETIMEOUT) or failed a device-side check."""
+        for A in self._arenas:
+            if A is not None and A.ws is not None:
+                G.gefen_step_status(A.ws)
+            if A is not None and A.rws is not None:
+                G.gefen_refit_status(A.rws)
+
+    # --------------------------------------------------- checkpointing
+    def state_dict(self):
+        sd = super().state_dict()
+        groups = []
+        for A in self._arenas:
+            if A is None:
+                groups.append(None)
+                continue
+            groups.append(dict(t=A.t, periods=list(A.periods), switch=A.switch,
+                               codes=A.codes.clone(), v=A.v.clone(), s=A.s.clone(),
+                               cb=A.cb.clone(), cb_new=A.cb_new.clone()))
+        sd["gefen"] = dict(levels=self.levels, bins=self.bins, refit_every=self.refit_every, groups=groups)
+        return sd
+
+    def load_state_dict(self, state_dict):
+        state_dict = dict(state_dict)
+        gst = state_dict.pop("gefen", None)
+        super().load_state_dict(state_dict)
+        if gst is None:
+            return
+        if gst["levels"] != self.levels or gst["bins"] != self.bins:
+            raise ValueError("checkpoint was written with another codebook size or histogram")
+        self._pending = list(gst["groups"])
+        for gi, A in enumerate(self._arenas):
+            if A is not None and self._pending[gi] is not None:
+                self._restore(A, self._pending[gi])
+
+    @staticmethod
+    def _restore(A: _Arena, st: Dict):
+        A.set_periods(st["periods"])
+        A.t = int(st["t"])
+        A.switch = bool(st["switch"])
+        for name in ("codes", "v", "s", "cb", "cb_new"):
+            src = st[name]
+            dst = getattr(A, name)
+            if src.numel() != dst.numel():
+                raise ValueError(f"checkpoint {name} has {src.numel()} entries, expected {dst.numel()}")
+            dst.copy_(src.to(dst.device))

@@ -1,0 +1,121 @@
+"""The torch.optim wrapper (paper_2606_13894_gb300.optim.Gefen): each of its
+steps equals the oracle's step from the wrapper's own pre-step state (right
+hyper-parameters, step count, codebook switch after a refit), a checkpoint
+resumes bit for bit, and it trains a small regression."""
+import numpy as np
+import pytest
+import torch
+
+import gpu_util as U
+from paper_2606_13894_gb300.optim import Gefen
+
+pytestmark = pytest.mark.gpu
+
+
+def _model(seed=0):
+    torch.manual_seed(seed)
+    return torch.nn.Sequential(torch.nn.Linear(64, 256), torch.nn.ReLU(), torch.nn.Linear(256, 32)).cuda()
+
+
+def _batch(i):
+    g = torch.Generator(device="cuda").manual_seed(1000 + i)
+    x = torch.randn(128, 64, device="cuda", generator=g)
+    y = torch.randn(128, 32, device="cuda", generator=g)
+    return x, y
+
+
+def _backward(model, i):
+    x, y = _batch(i)
+    model.zero_grad(set_to_none=True)
+    loss = torch.nn.functional.mse_loss(model(x), y)
+    loss.backward()
+    return loss
+
+
+class _View:
+    """The comparison helpers' arena interface over the wrapper's arena."""
+
+    def __init__(self, A):
+        self.entries, self.NB = A.entries, A.v.numel()
+
+
+def test_each_wrapper_step_matches_the_oracle():
+    model = _model()
+    hp = dict(lr=3e-3, betas=(0.9, 0.99), eps=1e-8, weight_decay=0.05)
+    opt = Gefen(model.parameters(), **hp, refit_every=3)
+    ohp = dict(lr=hp["lr"], beta1=hp["betas"][0], beta2=hp["betas"][1], eps=hp["eps"], weight_decay=hp["weight_decay"])
+    for i in range(8):
+        _backward(model, i)
+        A = opt._arenas[0]
+        if A is None:  # the first step sets up blocks and the first codebook
+            opt.step()
+            A = opt._arenas[0]
+            assert A.t == 1 and all(p.data.data_ptr() >= A.theta.data_ptr() for p in model.parameters())
+            continue
+        pre = (A.theta.cpu().numpy().copy(), A.codes.cpu().numpy().copy(), A.v.cpu().numpy().copy(),
+               A.s.cpu().numpy().copy())
+        dec = A.cb.cpu().numpy().copy()
+        enc = (A.cb_new if A.switch else A.cb).cpu().numpy().copy()
+        opt.step()
+        gbits = U.bits(A.grads)
+        got = (A.theta.cpu().numpy(), A.codes.cpu().numpy(), A.v.cpu().numpy(), A.s.cpu().numpy())
+        V = _View(A)
+        th, cd, vv, ss, _ = U.oracle_step(V, pre, gbits, dec, enc, A.t, ohp)
+        assert U.theta_err(got[0], th, ohp["lr"]) <= U.THETA_TOL, i
+        assert U.rel_err(got[2], vv) <= U.STATE_TOL, i
+        M = U.summand_scale(V, pre, gbits, dec, ohp["beta1"])
+        assert U.scale_ok(got[3], ss, M)[0], i
+        assert U.code_flips_ok(V, pre, gbits, dec, enc, got[1], cd, ohp, M)[0], i
+    opt.check()
+
+
+def test_checkpoint_resumes_bit_for_bit():
+    m1 = _model(1)
+    o1 = Gefen(m1.parameters(), lr=2e-3, refit_every=2)
+    for i in range(5):
+        _backward(m1, i)
+        o1.step()
+    sd_m, sd_o = m1.state_dict(), o1.state_dict()
+    m2 = _model(2)
+    m2.load_state_dict(sd_m)
+    o2 = Gefen(m2.parameters(), lr=2e-3, refit_every=2)
+    o2.load_state_dict(sd_o)
+    for i in range(5, 9):
+        _backward(m1, i)
+        o1.step()
+        _backward(m2, i)
+        o2.step()
+    for a, b in zip(m1.parameters(), m2.parameters()):
+        assert torch.equal(a, b)
+
+
+def test_trains_a_regression():
+    torch.manual_seed(3)
+    w_true = torch.randn(64, 8, device="cuda")
+    model = torch.nn.Linear(64, 8, bias=False).cuda()
+    opt = Gefen(model.parameters(), lr=3e-2, weight_decay=0.0, refit_every=10)
+    losses = []
+    for i in range(60):
+        g = torch.Generator(device="cuda").manual_seed(i)
+        x = torch.randn(256, 64, device="cuda", generator=g)
+        model.zero_grad(set_to_none=True)
+        loss = torch.nn.functional.mse_loss(model(x), x @ w_true)
+        loss.backward()
+        opt.step()
+        losses.append(float(loss.detach()))
+    assert losses[-1] < 0.1 * losses[0]
+
+
+def test_parameters_without_grad_are_untouched():
+    model = _model(4)
+    opt = Gefen(model.parameters(), lr=1e-2)
+    _backward(model, 0)
+    opt.step()
+    frozen = model[2].weight.detach().clone()
+    model[2].weight.requires_grad_(False)
+    x, y = _batch(1)
+    model.zero_grad(set_to_none=True)
+    torch.nn.functional.mse_loss(model(x), y).backward()
+    assert model[2].weight.grad is None
+    opt.step()
+    assert torch.equal(model[2].weight, frozen)
