@@ -49,8 +49,10 @@ struct Seg {
     int64_t aux_begin;   // big path: first big-block index of this tensor
     int64_t nblocks;     // numel / period
     uint32_t pmagic;     // floor(2^32 / period) + 1: e / p == umulhi(e, pmagic) for e * p < 2^32
-    uint32_t pad;
+    uint32_t flags;  // kSegBigTiles: tiles of big blocks whose factors come from blk_state
 };
+
+constexpr uint32_t kSegBigTiles = 1u;
 
 inline void seg_fill(Seg& s, const gefen_tensor_t& x) {
     s.elem_off = x.offset;
@@ -59,7 +61,7 @@ inline void seg_fill(Seg& s, const gefen_tensor_t& x) {
     s.block_off = x.block_offset;
     s.nblocks = x.numel / x.period;
     s.pmagic = static_cast<uint32_t>((uint64_t(1) << 32) / static_cast<uint64_t>(x.period)) + 1u;
-    s.pad = 0;
+    s.flags = 0;
 }
 
 struct HP {
@@ -397,11 +399,13 @@ constexpr float kLutGuard = 2.384185791015625e-07f;  // 2^-22, below every cell 
 
 struct TileInfo {
     int64_t e0;    // first element
-    int64_t bo;    // first block index into v / scale
+    int64_t bo;    // first block index into v / scale (big-block tiles: index into blk_state)
     int nelem;
     int nblk;
     int p;
     uint32_t pmagic;  // floor(2^32 / p) + 1: e / p == umulhi(e, pmagic) for e, p < 2^16
+    int ext;          // a tile of a big block: its factors were finalised beforehand
+    int pad;
 };
 
 template <int LUTR, int DECR>
@@ -503,8 +507,23 @@ __device__ __forceinline__ TileInfo tile_info(const Launch& L, int64_t unit, int
     while (seg + 1 < L.nseg && L.seg[seg + 1].unit_begin <= unit) ++seg;
     const Seg& S = L.seg[seg];
     const int64_t p = S.period;
-    const int64_t blk0 = (unit - S.unit_begin) * S.per_unit;
     TileInfo ti;
+    ti.pad = 0;
+    if (S.flags & kSegBigTiles) {
+        // per_unit tiles per block, each p / per_unit consecutive elements
+        const int64_t local = unit - S.unit_begin;
+        const int64_t tsz = p / S.per_unit;
+        ti.ext = 1;
+        ti.nblk = 1;
+        ti.p = static_cast<int>(min(p, static_cast<int64_t>(1) << 30));
+        ti.nelem = static_cast<int>(tsz);
+        ti.e0 = S.elem_off + local * tsz;
+        ti.bo = S.aux_begin + local / S.per_unit;
+        ti.pmagic = 0u;
+        return ti;
+    }
+    ti.ext = 0;
+    const int64_t blk0 = (unit - S.unit_begin) * S.per_unit;
     ti.nblk = static_cast<int>(min(S.per_unit, S.nblocks - blk0));
     ti.p = static_cast<int>(p);
     ti.nelem = ti.nblk * ti.p;
@@ -546,6 +565,12 @@ __device__ __forceinline__ void issue_tile(Smem& sm, int s, const TileInfo& ti, 
 // groups, whose first elements are eb + 128 j.
 template <int NG>
 __device__ __forceinline__ void load_state(const Ptrs& P, const TileInfo& ti, int eb, float (&s)[NG], float (&v)[NG]) {
+    if (ti.ext) {  // a big block: s before the step was kept by its finalisation
+        const float s0 = P.blk_state[ti.bo].x;
+#pragma unroll
+        for (int j = 0; j < NG; ++j) { s[j] = s0; v[j] = 0.0f; }
+        return;
+    }
     if (ti.p > 65535) return;              // only a tile that does not fit; never processed
     if (ti.p % (128 * NG) == 0) {          // one block per warp slice
         if (eb < ti.nelem) {
@@ -681,7 +706,13 @@ __device__ __forceinline__ void stream_tile(Smem& sm, const Ptrs& P, const HP& h
             }
         }
     };
-    if ((p & 511) == 0) {
+    if (ti.ext) {
+        // a tile of a big block: v, s and the step factor were finalised
+        const float4 bs = P.blk_state[ti.bo];  // (s before, s after, step factor, -)
+        const float iv = (MODE == kGradOnly) ? bs.y : (bs.y > 0.0f ? __frcp_rn(bs.y) : 0.0f);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) { fac[j] = bs.z; inv[j] = iv; }
+    } else if ((p & 511) == 0) {
         // a warp's 512 elements lie in one block
         float s2 = (g2[0] + g2[1]) + (g2[2] + g2[3]);
         float sx = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
@@ -1343,9 +1374,9 @@ cudaError_t launch_class(K kernel, Launch& L, const std::vector<int>& ids, const
     return cudaSuccess;
 }
 
+// One launch of the streamed kernel over the units of a prepared Launch.
 template <typename C, int MODE, int HB>
-cudaError_t launch_stream(Launch& L, const std::vector<int>& ids, const gefen_tensor_t* t, PathClass c,
-                          const Ptrs& P, int* err, cudaStream_t st) {
+cudaError_t stream_kernel(const Launch& L, const Ptrs& P, int* err, cudaStream_t st) {
     auto kern = k_step_stream<C::TILE, C::THREADS, C::STAGES, C::LUTR, C::DECR, C::THS, HB, MODE, C::MINB>;
     const int smem = static_cast<int>(sizeof(StreamSmem<C::TILE, C::THREADS, C::STAGES, C::LUTR, C::DECR, C::THS, HB>));
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
@@ -1356,12 +1387,25 @@ cudaError_t launch_stream(Launch& L, const std::vector<int>& ids, const gefen_te
     e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, C::THREADS, smem);
     if (e != cudaSuccess) return e;
     const int64_t cap = static_cast<int64_t>(std::max(1, per_sm)) * device_sm_count();
-    return launch_class(
-        [&](Launch& LL, int64_t u) {
-            kern<<<dim3(static_cast<unsigned>(std::min(u, cap))), C::THREADS, smem, st>>>(LL, P, err);
+    kern<<<dim3(static_cast<unsigned>(std::min(L.nunits, cap))), C::THREADS, smem, st>>>(L, P, err);
+    return cudaGetLastError();
+}
+
+template <typename C, int MODE, int HB>
+cudaError_t launch_stream(Launch& L, const std::vector<int>& ids, const gefen_tensor_t* t, PathClass c,
+                          const Ptrs& P, int* err, cudaStream_t st) {
+    cudaError_t e2 = cudaSuccess;
+    cudaError_t e = launch_class(
+        [&](Launch& LL, int64_t) {
+            if (e2 == cudaSuccess) e2 = stream_kernel<C, MODE, HB>(LL, P, err, st);
         },
         L, ids, t, c, C::TILE);
+    return e != cudaSuccess ? e : e2;
 }
+
+// Big blocks whose size is a multiple of the streamed tile are applied by the
+// streamed kernel, tile by tile, with the factors their finalisation kept.
+inline bool big_streamable(int64_t p) { return p > kTile16Max && p % kS4KTile == 0; }
 
 // fused: the streamed kernels count the histogram in shared memory (the
 // other kernels stage x for launch_histogram).
@@ -1410,7 +1454,35 @@ cudaError_t run_step(const Plan& pl, const gefen_tensor_t* t, Launch& L, const P
             if (units == 0) continue;
             k_big_partial<MODE><<<dim3(units), kThreads, 0, st>>>(L, P, aligned);
             k_big_finalize<MODE><<<dim3(blocks), kThreads, 0, st>>>(L, P);
-            k_big_apply<MODE><<<dim3(units), kThreads, 0, st>>>(L, P, aligned);
+            if ((e = cudaGetLastError()) != cudaSuccess) return e;
+            // apply: streamed tiles where the block size allows, chunks otherwise
+            // (same big-block numbering, so both read the finalised state)
+            static thread_local Launch LS, LA;
+            LS.hp = LA.hp = L.hp;
+            LS.nseg = LA.nseg = 0;
+            LS.nunits = LA.nunits = 0;
+            for (int j = 0; j < L.nseg; ++j) {
+                const Seg& sj = L.seg[j];
+                if (big_streamable(sj.period)) {
+                    Seg& d = LS.seg[LS.nseg++];
+                    d = sj;
+                    d.flags = kSegBigTiles;
+                    d.per_unit = sj.period / kS4KTile;
+                    d.unit_begin = LS.nunits;
+                    LS.nunits += sj.nblocks * d.per_unit;
+                } else {
+                    Seg& d = LA.seg[LA.nseg++];
+                    d = sj;
+                    d.unit_begin = LA.nunits;
+                    LA.nunits += sj.nblocks * sj.per_unit;
+                }
+            }
+            if (LS.nunits > 0) {
+                e = (MODE != kPlain && fused) ? stream_kernel<S4KHistCfg, MODE, kFusedBins>(LS, P, err, st)
+                                              : stream_kernel<S4KCfg, MODE, 0>(LS, P, err, st);
+                if (e != cudaSuccess) return e;
+            }
+            if (LA.nunits > 0) k_big_apply<MODE><<<dim3(LA.nunits), kThreads, 0, st>>>(LA, P, aligned);
             if ((e = cudaGetLastError()) != cudaSuccess) return e;
         }
     }
@@ -1501,7 +1573,8 @@ extern "C" gefen_status_t gefen_step(const gefen_tensor_t* tensors, int32_t nten
         for (int i = 0; i < ntensors; ++i) {
             if (tensors[i].numel == 0) continue;
             const PathClass c = classify(tensors[i].period);
-            if (fused && (c == kS4K || c == kS8K)) continue;  // counted in place
+            if (fused && (c == kS4K || c == kS8K || (c == kBigAligned && big_streamable(tensors[i].period))))
+                continue;  // counted in place
             rr.push_back({tensors[i].offset, tensors[i].numel});
         }
         if (!rr.empty() && launch_histogram(P.xstage, rr.data(), static_cast<int>(rr.size()), hist_bins, hist, st) !=
