@@ -844,24 +844,27 @@ __device__ __forceinline__ void stream_loop(Smem& sm, const Launch& L, const Ptr
         const int s = it % STAGES;
         const uint32_t parity = static_cast<uint32_t>((it / STAGES) & 1);
         const TileInfo ti = sm.tile[s];
-        const bool fits = tile_fits<TILE>(ti);
-        const bool ok = fits ? mbar_wait(smem_u32(&sm.bar[s]), parity) : true;
-        if (__syncthreads_or(!fits || !ok)) {
-            // A tile the host planned too large (nothing was copied for it) or
-            // a copy that never completed: wait, bounded, for the copies still
-            // in flight, flag the error and stop.
-            for (int j = fits ? 0 : 1; j < STAGES; ++j) {
+        if (!tile_fits<TILE>(ti)) {
+            // a tile the host planned too large (uniform: every thread reads
+            // the same descriptor): nothing was copied for it.  Wait, bounded,
+            // for the copies already issued for later tiles, flag, stop.
+            __syncthreads();  // descriptors the issuing thread wrote since the last barrier
+            for (int j = 1; j < STAGES; ++j) {
                 const int64_t uj = u + static_cast<int64_t>(j) * G;
                 if (uj >= L.nunits || !tile_fits<TILE>(sm.tile[(it + j) % STAGES])) continue;
                 mbar_wait(smem_u32(&sm.bar[(it + j) % STAGES]), static_cast<uint32_t>(((it + j) / STAGES) & 1));
             }
-            if (tid == 0) atomicExch(err, fits ? 1 : 2);
+            if (tid == 0) atomicExch(err, 2);
             break;
         }
-        // block state of the next tile, one tile ahead (its descriptor was
-        // published before the barrier above)
+        // each thread waits for the stage itself; a wait that gives up is
+        // acted on, uniformly, at the end of the tile
+        const bool ok = mbar_wait(smem_u32(&sm.bar[s]), parity);
+        // block state of the next tile, one tile ahead: with three or more
+        // stages its descriptor was published before the last barrier
         float n_s[4] = {0.0f, 0.0f, 0.0f, 0.0f}, n_v[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-        if (MODE != kGradOnly && u + G < L.nunits) load_state<4>(P, sm.tile[(it + 1) % STAGES], eb, n_s, n_v);
+        if (STAGES >= 3 && MODE != kGradOnly && u + G < L.nunits)
+            load_state<4>(P, sm.tile[(it + 1) % STAGES], eb, n_s, n_v);
 
         if (ti.nelem == TILE)
             stream_tile<TILE, THREADS, LUTR, DECR, MODE, THS, LUT, true>(sm, P, L.hp, ti, sm.stage[s], eb, r_s, r_v);
@@ -869,11 +872,23 @@ __device__ __forceinline__ void stream_loop(Smem& sm, const Launch& L, const Ptr
             stream_tile<TILE, THREADS, LUTR, DECR, MODE, THS, LUT, false>(sm, P, L.hp, ti, sm.stage[s], eb, r_s, r_v);
 
         // every thread is done with stage s: refill it with tile it + STAGES
-        __syncthreads();
+        if (__syncthreads_or(!ok)) {
+            // a copy that never completed (the tile's outputs are undefined):
+            // wait, bounded, for the copies still in flight, flag, stop
+            for (int j = 0; j < STAGES; ++j) {
+                const int64_t uj = u + static_cast<int64_t>(j) * G;
+                if (uj >= L.nunits || !tile_fits<TILE>(sm.tile[(it + j) % STAGES])) continue;
+                mbar_wait(smem_u32(&sm.bar[(it + j) % STAGES]), static_cast<uint32_t>(((it + j) / STAGES) & 1));
+            }
+            if (tid == 0) atomicExch(err, 1);
+            break;
+        }
         if (tid == 0) {
             const int64_t un = u + static_cast<int64_t>(STAGES) * G;
             if (un < L.nunits) issue_tile<TILE, MODE, THS>(sm, s, tile_info(L, un, seg), P);
         }
+        if (STAGES < 3 && MODE != kGradOnly && u + G < L.nunits)
+            load_state<4>(P, sm.tile[(it + 1) % STAGES], eb, n_s, n_v);
 #pragma unroll
         for (int j = 0; j < 4; ++j) { r_s[j] = n_s[j]; r_v[j] = n_v[j]; }
     }
