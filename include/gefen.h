@@ -61,7 +61,8 @@ typedef struct {
 
 /* Hyperparameters of Algorithm 1 (AdamW's: stepsize alpha = lr, weight decay
  * lambda, decay rates beta1, beta2 in [0,1), eps) and the step counter t >= 1
- * used by both bias corrections.  flags: see GEFEN_HIST*. */
+ * used by both bias corrections.  flags: GEFEN_HIST* and the storage formats
+ * GEFEN_CODES_4BIT, GEFEN_PARAMS_BF16 (below). */
 typedef struct {
     double lr;
     double beta1;
@@ -78,6 +79,18 @@ typedef struct {
 /* Only histogram g_i / max_{j in block}|g_j| of every nonzero block and write
  * nothing else: the histogram of Algorithm 3 built from the first gradient. */
 #define GEFEN_HIST_GRAD_ONLY 2u
+/* Storage formats (the four-bit codes of the Ablation Study, "Getting Down to
+ * Four Bits", and the 16-bit parameters of the mixed-precision runs in the
+ * Experiments; the arithmetic stays fp32):
+ * GEFEN_CODES_4BIT: k <= 16 and two codes per byte -- element i of the arena
+ * in byte i/2, the low nibble for even i; every tensor offset a multiple of
+ * 32.  GEFEN_PARAMS_BF16: params holds bf16 values (the update is computed in
+ * fp32 and rounded to nearest-even).  Either format is available for blocks
+ * of 1 element, blocks of p <= 8192 with p % 16 == 0 (p % 32 == 0 with 4-bit
+ * codes) and larger blocks with p % 4096 == 0; other tensors, and histograms
+ * of more than 4096 cells, return GEFEN_EUNSUPPORTED. */
+#define GEFEN_CODES_4BIT 4u
+#define GEFEN_PARAMS_BF16 8u
 
 /* Largest histogram supported by every call (bins), and largest codebook. */
 #define GEFEN_MAX_BINS 65536
@@ -106,8 +119,10 @@ gefen_status_t gefen_sync_status(gefen_stream_t stream);
  * codebook refit, pass the old codebook as codebook_dec and the new one as
  * codebook_enc for one step.
  *
- * params  f32[*]  device, in/out     grads  bf16[*] device, in
- * codes   u8[*]   device, in/out     v, scale f32[*] device, in/out (per block)
+ * params  f32[*] (bf16 with GEFEN_PARAMS_BF16) device, in/out
+ * grads   bf16[*] device, in
+ * codes   u8[*] (two per byte with GEFEN_CODES_4BIT) device, in/out
+ * v, scale f32[*] device, in/out (per block)
  * codebook_dec, codebook_enc  f32[k] device, sorted ascending, 2 <= k <= 256
  * hist    u64[hist_bins] device, counts are ADDED (caller zeroes); required
  *         when a GEFEN_HIST* flag is set, else ignored (may be NULL).

@@ -24,6 +24,8 @@
 #include <cstring>
 #include <vector>
 
+#include <cuda_bf16.h>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -38,6 +40,68 @@ constexpr int kChunk = 8192;        // elements per CTA in the big-block path
 constexpr int64_t kTile16Max = 16384;
 
 enum Mode { kPlain = 0, kHist = 1, kGradOnly = 2 };
+
+// Storage formats: bit 0 = two 4-bit codes per byte (element i in byte i/2,
+// low nibble for even i), bit 1 = bf16 theta.  The arithmetic is fp32 in all.
+template <int FMT>
+struct Format {
+    static constexpr bool kC4 = (FMT & 1) != 0;
+    static constexpr bool kTB = (FMT & 2) != 0;
+    static constexpr int kThetaBytes = kTB ? 2 : 4;
+};
+
+// The four codes of a group of four elements starting at element e (e % 4 == 0).
+template <int FMT>
+__device__ __forceinline__ uint32_t codes4_at(const unsigned char* base, int64_t e) {
+    if (Format<FMT>::kC4) return *reinterpret_cast<const uint16_t*>(base + (e >> 1));
+    return *reinterpret_cast<const uint32_t*>(base + e);
+}
+template <int FMT>
+__device__ __forceinline__ uint32_t code_of(uint32_t w, int i) {
+    if (Format<FMT>::kC4) return (w >> (4 * i)) & 0xFu;
+    return __byte_perm(w, 0u, 0x4440u + i);
+}
+template <int FMT>
+__device__ __forceinline__ uint32_t pack_codes4(const uint32_t (&c)[4]) {
+    if (Format<FMT>::kC4) return c[0] | (c[1] << 4) | (c[2] << 8) | (c[3] << 12);
+    return __byte_perm(__byte_perm(c[0], c[1], 0x0040u), __byte_perm(c[2], c[3], 0x0040u), 0x5410u);
+}
+template <int FMT>
+__device__ __forceinline__ void store_codes4(uint8_t* codes, int64_t e, uint32_t packed) {
+    if (Format<FMT>::kC4)
+        __stcs(reinterpret_cast<unsigned short*>(codes + (e >> 1)), static_cast<unsigned short>(packed));
+    else
+        __stcs(reinterpret_cast<unsigned int*>(codes + e), packed);
+}
+// Four theta values starting at element e of an fp32 or bf16 array.
+template <int FMT>
+__device__ __forceinline__ float4 theta4_global(const float* params, int64_t e) {
+    if (Format<FMT>::kTB) {
+        const uint2 w = __ldcs(reinterpret_cast<const uint2*>(reinterpret_cast<const uint16_t*>(params) + e));
+        return make_float4(bf16_lo(w.x), bf16_hi(w.x), bf16_lo(w.y), bf16_hi(w.y));
+    }
+    return __ldcs(reinterpret_cast<const float4*>(params + e));
+}
+template <int FMT>
+__device__ __forceinline__ float4 theta4_smem(const unsigned char* base, int e) {
+    if (Format<FMT>::kTB) {
+        const uint2 w = *reinterpret_cast<const uint2*>(base + 2 * e);
+        return make_float4(bf16_lo(w.x), bf16_hi(w.x), bf16_lo(w.y), bf16_hi(w.y));
+    }
+    return *reinterpret_cast<const float4*>(base + 4 * e);
+}
+__device__ __forceinline__ uint32_t bf16_pair_rn(float lo, float hi) {
+    const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);  // .x = lo (low half), .y = hi
+    return *reinterpret_cast<const uint32_t*>(&v);
+}
+template <int FMT>
+__device__ __forceinline__ void theta4_store(float* params, int64_t e, float4 t) {
+    if (Format<FMT>::kTB)
+        __stcs(reinterpret_cast<uint2*>(reinterpret_cast<uint16_t*>(params) + e),
+               make_uint2(bf16_pair_rn(t.x, t.y), bf16_pair_rn(t.z, t.w)));
+    else
+        __stcs(reinterpret_cast<float4*>(params + e), t);
+}
 
 struct Seg {
     int64_t elem_off;
@@ -164,44 +228,64 @@ __device__ __forceinline__ uint32_t byte_of(uint4 c, int i) {
 
 // ------------------------------------------------------------------ p == 1
 // Every element is its own block: v and s are per element, x = m/|m| = +-1.
-template <int MODE>
+// With two codes per byte a thread owns both elements of a byte (a pair);
+// the nibble of an element past the tensor's end is left as it was.
+template <int MODE, int FMT>
 __global__ void __launch_bounds__(kThreads) k_step_p1(const __grid_constant__ Launch L, const Ptrs P) {
+    constexpr int EPC = Format<FMT>::kC4 ? 2 : 1;  // elements per thread and step
     __shared__ float s_dec[kMaxLevels], s_mid[kMaxLevels];
     if (MODE != kGradOnly) load_codebooks(P, s_dec, s_mid);
     __syncthreads();
     const int64_t unit = blockIdx.x;
     const Seg& S = L.seg[find_seg(L, unit)];
-    const int64_t base = (unit - S.unit_begin) * (4 * kThreads);
+    const int64_t base = (unit - S.unit_begin) * (4 * kThreads * EPC);
     const HP& hp = L.hp;
     const int zero_code = (MODE != kGradOnly) ? level_search(s_mid, 0.0f) : 0;
+    uint16_t* th16 = reinterpret_cast<uint16_t*>(P.params);
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-        const int64_t le = base + threadIdx.x + i * kThreads;
-        if (le >= S.numel) break;
-        const int64_t e = S.elem_off + le;
-        const int64_t bi = S.block_off + le;
-        const float g = bf16_bits_to_f32(__ldcs(P.grads + e));
-        if (MODE == kGradOnly) {
-            P.xstage[e] = g != 0.0f ? __fdiv_rn(g, fabsf(g)) : __int_as_float(0x7fffffff);
-            continue;
+        const int64_t c0 = base + (threadIdx.x + i * kThreads) * static_cast<int64_t>(EPC);
+        if (c0 >= S.numel) break;
+        uint32_t cbyte = 0u;
+        if (MODE != kGradOnly && Format<FMT>::kC4) cbyte = P.codes[(S.elem_off + c0) >> 1];
+#pragma unroll
+        for (int q = 0; q < EPC; ++q) {
+            const int64_t le = c0 + q;
+            if (le >= S.numel) break;
+            const int64_t e = S.elem_off + le;
+            const int64_t bi = S.block_off + le;
+            const float g = bf16_bits_to_f32(__ldcs(P.grads + e));
+            if (MODE == kGradOnly) {
+                P.xstage[e] = g != 0.0f ? __fdiv_rn(g, fabsf(g)) : __int_as_float(0x7fffffff);
+                continue;
+            }
+            const uint32_t cold = Format<FMT>::kC4 ? ((cbyte >> (4 * q)) & 0xFu) : __ldcs(P.codes + e);
+            const float m = fmaf(hp.omb1, g, hp.beta1 * P.scale[bi] * s_dec[cold]);
+            const float fac = block_update(hp, P.v, bi, g * g);
+            const float am = fabsf(m);
+            P.scale[bi] = am;
+            const float th = Format<FMT>::kTB ? bf16_bits_to_f32(__ldcs(th16 + e)) : __ldcs(P.params + e);
+            const float tn = fmaf(-fac, m, hp.decay * th);
+            if (Format<FMT>::kTB)
+                __stcs(th16 + e, __bfloat16_as_ushort(__float2bfloat16_rn(tn)));
+            else
+                __stcs(P.params + e, tn);
+            float x;
+            int c;
+            if (am > 0.0f) {
+                x = __fdiv_rn(m, am);
+                c = level_search(s_mid, x);
+            } else {
+                x = __int_as_float(0x7fffffff);
+                c = zero_code;
+            }
+            if (Format<FMT>::kC4)
+                cbyte = (cbyte & ~(0xFu << (4 * q))) | (static_cast<uint32_t>(c) << (4 * q));
+            else
+                P.codes[e] = static_cast<uint8_t>(c);
+            if (MODE == kHist) P.xstage[e] = x;
         }
-        const float m = fmaf(hp.omb1, g, hp.beta1 * P.scale[bi] * s_dec[__ldcs(P.codes + e)]);
-        const float fac = block_update(hp, P.v, bi, g * g);
-        const float am = fabsf(m);
-        P.scale[bi] = am;
-        const float th = __ldcs(P.params + e);
-        __stcs(P.params + e, fmaf(-fac, m, hp.decay * th));
-        float x;
-        int c;
-        if (am > 0.0f) {
-            x = __fdiv_rn(m, am);
-            c = level_search(s_mid, x);
-        } else {
-            x = __int_as_float(0x7fffffff);
-            c = zero_code;
-        }
-        P.codes[e] = static_cast<uint8_t>(c);
-        if (MODE == kHist) P.xstage[e] = x;
+        if (MODE != kGradOnly && Format<FMT>::kC4) P.codes[(S.elem_off + c0) >> 1] = static_cast<uint8_t>(cbyte);
     }
 }
 
@@ -415,18 +499,18 @@ struct alignas(16) StreamTables {
     float mid[kMaxLevels + 4];
 };
 
-// Stage layout: [theta f32 (THS only) | g bf16 | codes u8].
-template <int TILE, bool THS>
+// Stage layout: [theta (THS only) | g bf16 | codes].
+template <int TILE, bool THS, int FMT>
 struct StageLayout {
-    static constexpr int kG = THS ? 4 * TILE : 0;
+    static constexpr int kG = THS ? Format<FMT>::kThetaBytes * TILE : 0;
     static constexpr int kC = kG + 2 * TILE;
-    static constexpr int kBytes = kC + TILE;
+    static constexpr int kBytes = kC + (Format<FMT>::kC4 ? TILE / 2 : TILE);
 };
 
-template <int TILE, int THREADS, int STAGES, int LUTR, int DECR, bool THS, int HB>
+template <int TILE, int THREADS, int STAGES, int LUTR, int DECR, bool THS, int HB, int FMT>
 struct alignas(128) StreamSmem {
     static constexpr int kHistCells = HB;  // cells counted in shared memory (0: x is staged instead)
-    unsigned char stage[STAGES][StageLayout<TILE, THS>::kBytes];
+    unsigned char stage[STAGES][StageLayout<TILE, THS, FMT>::kBytes];
     uint32_t hist[HB > 0 ? HB : 1];
     StreamTables<LUTR, DECR> tab;
     float2 part[THREADS / 32];  // per warp: (sum g^2, max |m|)
@@ -541,9 +625,10 @@ __device__ __forceinline__ bool tile_fits(const TileInfo& ti) {
 }
 
 // Publishes the tile's descriptor in its stage and starts its copies.
-template <int TILE, int MODE, bool THS, typename Smem>
+template <int TILE, int MODE, bool THS, int FMT, typename Smem>
 __device__ __forceinline__ void issue_tile(Smem& sm, int s, const TileInfo& ti, const Ptrs& P) {
-    using SL = StageLayout<TILE, THS>;
+    using SL = StageLayout<TILE, THS, FMT>;
+    constexpr uint32_t TB = Format<FMT>::kThetaBytes;
     sm.tile[s] = ti;
     if (!tile_fits<TILE>(ti)) return;  // never copied; the consumer stops before waiting on it
     const uint32_t n = static_cast<uint32_t>(ti.nelem);
@@ -553,11 +638,16 @@ __device__ __forceinline__ void issue_tile(Smem& sm, int s, const TileInfo& ti, 
         mbar_expect_tx(bar, 2u * n);
         bulk_g2s(smem_u32(st + SL::kG), P.grads + ti.e0, 2u * n, bar);
     } else {
-        mbar_expect_tx(bar, (THS ? 7u : 3u) * n);
-        if (THS) bulk_g2s(smem_u32(st), P.params + ti.e0, 4u * n, bar);
+        // codes: n bytes, or n/2 with two per byte (tiles start and end on
+        // multiples of 32 elements then, so every copy is whole 16-byte units)
+        const uint32_t cn = Format<FMT>::kC4 ? n / 2 : n;
+        const unsigned char* cs = P.codes + (Format<FMT>::kC4 ? ti.e0 / 2 : ti.e0);
+        const unsigned char* ts = reinterpret_cast<const unsigned char*>(P.params) + TB * ti.e0;
+        mbar_expect_tx(bar, (THS ? TB * n : 0u) + 2u * n + cn);
+        if (THS) bulk_g2s(smem_u32(st), ts, TB * n, bar);
         bulk_g2s(smem_u32(st + SL::kG), P.grads + ti.e0, 2u * n, bar);
-        bulk_g2s(smem_u32(st + SL::kC), P.codes + ti.e0, n, bar);
-        if (!THS) prefetch_l2(P.params + ti.e0, 4u * n);
+        bulk_g2s(smem_u32(st + SL::kC), cs, cn, bar);
+        if (!THS) prefetch_l2(ts, TB * n);
     }
 }
 
@@ -614,9 +704,9 @@ __device__ __forceinline__ uint32_t lt_mask(float a, float b) {
 // bit pattern of y minus that of 1.5 * 2^23.  The unsigned clamp keeps a NaN
 // or a corrupted value inside the table.
 template <bool LUT, int LUTR, int DECR>
-__device__ __forceinline__ uint32_t encode4(const StreamTables<LUTR, DECR>& T, int copy, const float (&x)[4]) {
+__device__ __forceinline__ void encode4(const StreamTables<LUTR, DECR>& T, int copy, const float (&x)[4],
+                                        uint32_t (&c)[4]) {
     constexpr float kMagic = 12582912.0f;  // 1.5 * 2^23, bits 0x4B400000
-    uint32_t c[4];
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
         if (LUT) {
@@ -629,15 +719,14 @@ __device__ __forceinline__ uint32_t encode4(const StreamTables<LUTR, DECR>& T, i
             c[i] = static_cast<uint32_t>(level_search(T.mid, x[i]));
         }
     }
-    return __byte_perm(__byte_perm(c[0], c[1], 0x0040u), __byte_perm(c[2], c[3], 0x0040u), 0x5410u);
 }
 
 // One tile of the streamed step.  FULL: every group of the tile is live (the
 // tile holds TILE elements), so no group needs a bounds predicate.
-template <int TILE, int THREADS, int LUTR, int DECR, int MODE, bool THS, bool LUT, bool FULL, typename Smem>
+template <int TILE, int THREADS, int LUTR, int DECR, int MODE, bool THS, int FMT, bool LUT, bool FULL, typename Smem>
 __device__ __forceinline__ void stream_tile(Smem& sm, const Ptrs& P, const HP& hp, const TileInfo& ti,
                                             unsigned char* st, int eb, const float (&r_s)[4], const float (&r_v)[4]) {
-    using SL = StageLayout<TILE, THS>;
+    using SL = StageLayout<TILE, THS, FMT>;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int lut_copy = lane % LUTR, dec_copy = lane % DECR;
     const int p = ti.p;
@@ -650,12 +739,12 @@ __device__ __forceinline__ void stream_tile(Smem& sm, const Ptrs& P, const HP& h
         live[j] = FULL || e < ti.nelem;
         blk[j] = static_cast<int>(__umulhi(static_cast<uint32_t>(e), ti.pmagic));
     }
-    float* thp = P.params + ti.e0 + eb;  // group j at + 128 j
+    const int64_t ge0 = ti.e0 + eb;  // element of group 0; group j at + 128 j
     float4 th[4];  // theta from global memory is loaded early; from the stage, just before use
     if (MODE != kGradOnly && !THS) {
 #pragma unroll
         for (int j = 0; j < 4; ++j)
-            if (live[j]) th[j] = __ldcs(reinterpret_cast<const float4*>(thp + 128 * j));
+            if (live[j]) th[j] = theta4_global<FMT>(P.params, ge0 + 128 * j);
     }
 
     // phase 1: decode m, partials per group of four
@@ -675,11 +764,11 @@ __device__ __forceinline__ void stream_tile(Smem& sm, const Ptrs& P, const HP& h
                 mx[j] = fmaxf(mx[j], fabsf(g[i]));
             }
         } else {
-            const uint32_t cw = live[j] ? *reinterpret_cast<const uint32_t*>(st + SL::kC + e) : 0u;
+            const uint32_t cw = live[j] ? codes4_at<FMT>(st + SL::kC, e) : 0u;
             const float b1s = hp.beta1 * r_s[j];
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
-                const uint32_t c = __byte_perm(cw, 0u, 0x4440u + i);
+                const uint32_t c = code_of<FMT>(cw, i);
                 const float mm = fmaf(hp.omb1, g[i], b1s * dec[c * DECR]);
                 m[4 * j + i] = mm;
                 g2[j] = fmaf(g[i], g[i], g2[j]);
@@ -789,7 +878,6 @@ __device__ __forceinline__ void stream_tile(Smem& sm, const Ptrs& P, const HP& h
     // phase 2: theta', the new codes (and x for the histogram), stored
     // straight from registers.  A zero block (inv = 0) encodes x = 0, the
     // level nearest 0, and stages NaN for the histogram.
-    uint8_t* cdp = P.codes + ti.e0 + eb;
     float* xsp = (MODE != kPlain && Smem::kHistCells == 0) ? P.xstage + ti.e0 + eb : nullptr;
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
@@ -800,15 +888,17 @@ __device__ __forceinline__ void stream_tile(Smem& sm, const Ptrs& P, const HP& h
             for (int i = 0; i < 4; ++i)
                 x[i] = inv[j] > 0.0f ? __fdiv_rn(m[4 * j + i], inv[j]) : __int_as_float(0x7fffffff);
         } else {
-            float4 t = THS ? *reinterpret_cast<const float4*>(st + 4 * (eb + 128 * j)) : th[j];
+            float4 t = THS ? theta4_smem<FMT>(st, eb + 128 * j) : th[j];
             t.x = fmaf(-fac[j], m[4 * j], hp.decay * t.x);
             t.y = fmaf(-fac[j], m[4 * j + 1], hp.decay * t.y);
             t.z = fmaf(-fac[j], m[4 * j + 2], hp.decay * t.z);
             t.w = fmaf(-fac[j], m[4 * j + 3], hp.decay * t.w);
-            __stcs(reinterpret_cast<float4*>(thp + 128 * j), t);
+            theta4_store<FMT>(P.params, ge0 + 128 * j, t);
 #pragma unroll
             for (int i = 0; i < 4; ++i) x[i] = m[4 * j + i] * inv[j];
-            __stcs(reinterpret_cast<unsigned int*>(cdp + 128 * j), encode4<LUT>(sm.tab, lut_copy, x));
+            uint32_t c[4];
+            encode4<LUT>(sm.tab, lut_copy, x, c);
+            store_codes4<FMT>(P.codes, ge0 + 128 * j, pack_codes4<FMT>(c));
             if (MODE == kHist) {
 #pragma unroll
                 for (int i = 0; i < 4; ++i) x[i] = inv[j] > 0.0f ? x[i] : __int_as_float(0x7fffffff);
@@ -829,7 +919,7 @@ __device__ __forceinline__ void stream_tile(Smem& sm, const Ptrs& P, const HP& h
     }
 }
 
-template <int TILE, int THREADS, int STAGES, int LUTR, int DECR, int MODE, bool THS, bool LUT, typename Smem>
+template <int TILE, int THREADS, int STAGES, int LUTR, int DECR, int MODE, bool THS, int FMT, bool LUT, typename Smem>
 __device__ __forceinline__ void stream_loop(Smem& sm, const Launch& L, const Ptrs& P, int* err, int seg) {
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int64_t G = gridDim.x;
@@ -867,9 +957,9 @@ __device__ __forceinline__ void stream_loop(Smem& sm, const Launch& L, const Ptr
             load_state<4>(P, sm.tile[(it + 1) % STAGES], eb, n_s, n_v);
 
         if (ti.nelem == TILE)
-            stream_tile<TILE, THREADS, LUTR, DECR, MODE, THS, LUT, true>(sm, P, L.hp, ti, sm.stage[s], eb, r_s, r_v);
+            stream_tile<TILE, THREADS, LUTR, DECR, MODE, THS, FMT, LUT, true>(sm, P, L.hp, ti, sm.stage[s], eb, r_s, r_v);
         else
-            stream_tile<TILE, THREADS, LUTR, DECR, MODE, THS, LUT, false>(sm, P, L.hp, ti, sm.stage[s], eb, r_s, r_v);
+            stream_tile<TILE, THREADS, LUTR, DECR, MODE, THS, FMT, LUT, false>(sm, P, L.hp, ti, sm.stage[s], eb, r_s, r_v);
 
         // every thread is done with stage s: refill it with tile it + STAGES
         if (__syncthreads_or(!ok)) {
@@ -885,7 +975,7 @@ __device__ __forceinline__ void stream_loop(Smem& sm, const Launch& L, const Ptr
         }
         if (tid == 0) {
             const int64_t un = u + static_cast<int64_t>(STAGES) * G;
-            if (un < L.nunits) issue_tile<TILE, MODE, THS>(sm, s, tile_info(L, un, seg), P);
+            if (un < L.nunits) issue_tile<TILE, MODE, THS, FMT>(sm, s, tile_info(L, un, seg), P);
         }
         if (STAGES < 3 && MODE != kGradOnly && u + G < L.nunits)
             load_state<4>(P, sm.tile[(it + 1) % STAGES], eb, n_s, n_v);
@@ -894,9 +984,9 @@ __device__ __forceinline__ void stream_loop(Smem& sm, const Launch& L, const Ptr
     }
 }
 
-template <int TILE, int THREADS, int STAGES, int LUTR, int DECR, bool THS, int HB, int MODE, int MINB>
+template <int TILE, int THREADS, int STAGES, int LUTR, int DECR, bool THS, int HB, int FMT, int MODE, int MINB>
 __global__ void __launch_bounds__(THREADS, MINB) k_step_stream(const __grid_constant__ Launch L, const Ptrs P, int* err) {
-    using Smem = StreamSmem<TILE, THREADS, STAGES, LUTR, DECR, THS, HB>;
+    using Smem = StreamSmem<TILE, THREADS, STAGES, LUTR, DECR, THS, HB, FMT>;
     static_assert(TILE == 16 * THREADS && THREADS % 32 == 0 && STAGES >= 2, "tile shape");
     static_assert(32 % LUTR == 0 && 32 % DECR == 0, "table copies");
     extern __shared__ __align__(128) unsigned char smem_raw[];
@@ -909,7 +999,7 @@ __global__ void __launch_bounds__(THREADS, MINB) k_step_stream(const __grid_cons
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         for (int s = 0; s < STAGES; ++s) {
             const int64_t u = blockIdx.x + s * G;
-            if (u < L.nunits) issue_tile<TILE, MODE, THS>(sm, s, tile_info(L, u, seg), P);
+            if (u < L.nunits) issue_tile<TILE, MODE, THS, FMT>(sm, s, tile_info(L, u, seg), P);
         }
     }
     if (HB > 0)
@@ -917,9 +1007,9 @@ __global__ void __launch_bounds__(THREADS, MINB) k_step_stream(const __grid_cons
     const int bad = build_tables<THREADS>(P, sm.tab, MODE == kGradOnly);
     const bool lut_ok = !__syncthreads_or(bad);
     if (MODE != kGradOnly && lut_ok)
-        stream_loop<TILE, THREADS, STAGES, LUTR, DECR, MODE, THS, true>(sm, L, P, err, seg);
+        stream_loop<TILE, THREADS, STAGES, LUTR, DECR, MODE, THS, FMT, true>(sm, L, P, err, seg);
     else
-        stream_loop<TILE, THREADS, STAGES, LUTR, DECR, MODE, THS, false>(sm, L, P, err, seg);
+        stream_loop<TILE, THREADS, STAGES, LUTR, DECR, MODE, THS, FMT, false>(sm, L, P, err, seg);
     if (HB > 0) {
         // add the CTA's counts to the histogram
         __syncthreads();
@@ -1075,7 +1165,7 @@ __device__ __forceinline__ void for_chunk_elems(int64_t c0, int64_t c1, bool ali
     }
 }
 
-template <int MODE>
+template <int MODE, int FMT>
 __global__ void __launch_bounds__(kThreads) k_big_partial(const __grid_constant__ Launch L, const Ptrs P, int aligned) {
     __shared__ float s_dec[kMaxLevels];
     __shared__ double s_red[kThreads / 32];
@@ -1098,10 +1188,19 @@ __global__ void __launch_bounds__(kThreads) k_big_partial(const __grid_constant_
 #pragma unroll
                 for (int t = 0; t < 16; ++t) mx = fmaxf(mx, fabsf(g[t]));
             } else {
-                const uint4 cw = __ldcg(reinterpret_cast<const uint4*>(P.codes + e));
+                uint32_t cv[16];
+                if (Format<FMT>::kC4) {
+                    const uint2 cw = __ldcg(reinterpret_cast<const uint2*>(P.codes + (e >> 1)));
+#pragma unroll
+                    for (int t = 0; t < 16; ++t) cv[t] = ((t < 8 ? cw.x : cw.y) >> (4 * (t & 7))) & 0xFu;
+                } else {
+                    const uint4 cw = __ldcg(reinterpret_cast<const uint4*>(P.codes + e));
+#pragma unroll
+                    for (int t = 0; t < 16; ++t) cv[t] = byte_of(cw, t);
+                }
 #pragma unroll
                 for (int t = 0; t < 16; ++t) {
-                    const float mm = fmaf(hp.omb1, g[t], b1s * s_dec[byte_of(cw, t)]);
+                    const float mm = fmaf(hp.omb1, g[t], b1s * s_dec[cv[t]]);
                     g2 = fmaf(g[t], g[t], g2);
                     mx = fmaxf(mx, fabsf(mm));
                 }
@@ -1271,7 +1370,9 @@ PathClass classify(int64_t p) {
     return (p % 16 == 0) ? kBigAligned : kBigUnaligned;
 }
 
-int64_t units_of(PathClass c, const gefen_tensor_t& t, int64_t* per_unit, int64_t tile_cap = 0) {
+// p1_epc: elements each thread of k_step_p1 handles per round (2 with two
+// codes per byte).
+int64_t units_of(PathClass c, const gefen_tensor_t& t, int64_t* per_unit, int64_t tile_cap = 0, int p1_epc = 1) {
     const int64_t p = t.period, nb = t.numel / p;
     if (tile_cap > 0) {  // streamed classes: whole blocks per tile of the kernel's own size
         *per_unit = std::max<int64_t>(1, tile_cap / p);
@@ -1280,7 +1381,7 @@ int64_t units_of(PathClass c, const gefen_tensor_t& t, int64_t* per_unit, int64_
     switch (c) {
         case kP1:
             *per_unit = 1;
-            return (t.numel + 4 * kThreads - 1) / (4 * kThreads);
+            return (t.numel + 4 * kThreads * p1_epc - 1) / (4 * kThreads * p1_epc);
         case kS4K:
         case kS8K:
         case kT16V4: {
@@ -1366,7 +1467,7 @@ bool validate_tensors(const gefen_tensor_t* t, int32_t n) {
 // per group through `kernel(L, units)`.
 template <typename K>
 cudaError_t launch_class(K kernel, Launch& L, const std::vector<int>& ids, const gefen_tensor_t* t,
-                         PathClass c, int64_t tile_cap = 0) {
+                         PathClass c, int64_t tile_cap = 0, int p1_epc = 1) {
     size_t i = 0;
     while (i < ids.size()) {
         L.nseg = 0;
@@ -1378,7 +1479,7 @@ cudaError_t launch_class(K kernel, Launch& L, const std::vector<int>& ids, const
             s.unit_begin = units;
             s.aux_begin = 0;
             if (tile_cap > 0 && x.period > tile_cap) return cudaErrorInvalidValue;  // planning error
-            units += units_of(c, x, &s.per_unit, tile_cap);
+            units += units_of(c, x, &s.per_unit, tile_cap, p1_epc);
         }
         L.nunits = units;
         if (units == 0) continue;
@@ -1390,10 +1491,11 @@ cudaError_t launch_class(K kernel, Launch& L, const std::vector<int>& ids, const
 }
 
 // One launch of the streamed kernel over the units of a prepared Launch.
-template <typename C, int MODE, int HB>
+template <typename C, int MODE, int HB, int FMT>
 cudaError_t stream_kernel(const Launch& L, const Ptrs& P, int* err, cudaStream_t st) {
-    auto kern = k_step_stream<C::TILE, C::THREADS, C::STAGES, C::LUTR, C::DECR, C::THS, HB, MODE, C::MINB>;
-    const int smem = static_cast<int>(sizeof(StreamSmem<C::TILE, C::THREADS, C::STAGES, C::LUTR, C::DECR, C::THS, HB>));
+    auto kern = k_step_stream<C::TILE, C::THREADS, C::STAGES, C::LUTR, C::DECR, C::THS, HB, FMT, MODE, C::MINB>;
+    const int smem =
+        static_cast<int>(sizeof(StreamSmem<C::TILE, C::THREADS, C::STAGES, C::LUTR, C::DECR, C::THS, HB, FMT>));
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
@@ -1406,13 +1508,13 @@ cudaError_t stream_kernel(const Launch& L, const Ptrs& P, int* err, cudaStream_t
     return cudaGetLastError();
 }
 
-template <typename C, int MODE, int HB>
+template <typename C, int MODE, int HB, int FMT>
 cudaError_t launch_stream(Launch& L, const std::vector<int>& ids, const gefen_tensor_t* t, PathClass c,
                           const Ptrs& P, int* err, cudaStream_t st) {
     cudaError_t e2 = cudaSuccess;
     cudaError_t e = launch_class(
         [&](Launch& LL, int64_t) {
-            if (e2 == cudaSuccess) e2 = stream_kernel<C, MODE, HB>(LL, P, err, st);
+            if (e2 == cudaSuccess) e2 = stream_kernel<C, MODE, HB, FMT>(LL, P, err, st);
         },
         L, ids, t, c, C::TILE);
     return e != cudaSuccess ? e : e2;
@@ -1423,30 +1525,36 @@ cudaError_t launch_stream(Launch& L, const std::vector<int>& ids, const gefen_te
 inline bool big_streamable(int64_t p) { return p > kTile16Max && p % kS4KTile == 0; }
 
 // fused: the streamed kernels count the histogram in shared memory (the
-// other kernels stage x for launch_histogram).
-template <int MODE>
+// other kernels stage x for launch_histogram).  FMT: storage format (only
+// the classes the host validated for it occur).
+template <int MODE, int FMT>
 cudaError_t run_step(const Plan& pl, const gefen_tensor_t* t, Launch& L, const Ptrs& P, int* err, cudaStream_t st,
                      bool fused) {
     cudaError_t e;
-    e = launch_class([&](Launch& LL, int64_t u) { k_step_p1<MODE><<<dim3(u), kThreads, 0, st>>>(LL, P); },
-                     L, pl.idx[kP1], t, kP1);
+    e = launch_class([&](Launch& LL, int64_t u) { k_step_p1<MODE, FMT><<<dim3(u), kThreads, 0, st>>>(LL, P); },
+                     L, pl.idx[kP1], t, kP1, 0, Format<FMT>::kC4 ? 2 : 1);
     if (e != cudaSuccess) return e;
-    if (MODE != kPlain && fused)
-        e = launch_stream<S4KHistCfg, MODE, kFusedBins>(L, pl.idx[kS4K], t, kS4K, P, err, st);
-    else
-        e = launch_stream<S4KCfg, MODE, 0>(L, pl.idx[kS4K], t, kS4K, P, err, st);
-    if (e != cudaSuccess) return e;
-    if (MODE != kPlain && fused)
-        e = launch_stream<S8KHistCfg, MODE, kFusedBins>(L, pl.idx[kS8K], t, kS8K, P, err, st);
-    else
-        e = launch_stream<S8KCfg, MODE, 0>(L, pl.idx[kS8K], t, kS8K, P, err, st);
-    if (e != cudaSuccess) return e;
-    e = launch_class([&](Launch& LL, int64_t u) { k_step_tile16<4, MODE><<<dim3(u), kThreads, 0, st>>>(LL, P); },
-                     L, pl.idx[kT16V4], t, kT16V4);
-    if (e != cudaSuccess) return e;
-    e = launch_class([&](Launch& LL, int64_t u) { k_step_generic<MODE><<<dim3(u), kThreads, 0, st>>>(LL, P); },
-                     L, pl.idx[kGeneric], t, kGeneric);
-    if (e != cudaSuccess) return e;
+    auto streamed = [&](auto cfg, auto hist_cfg, PathClass c) -> cudaError_t {
+        using C = decltype(cfg);
+        using CH = decltype(hist_cfg);
+        if constexpr (MODE != kPlain) {
+            if (fused) return launch_stream<CH, MODE, kFusedBins, FMT>(L, pl.idx[c], t, c, P, err, st);
+            if constexpr (FMT == 0) return launch_stream<C, MODE, 0, 0>(L, pl.idx[c], t, c, P, err, st);
+            return pl.idx[c].empty() ? cudaSuccess : cudaErrorNotSupported;
+        } else {
+            return launch_stream<C, MODE, 0, FMT>(L, pl.idx[c], t, c, P, err, st);
+        }
+    };
+    if ((e = streamed(S4KCfg{}, S4KHistCfg{}, kS4K)) != cudaSuccess) return e;
+    if ((e = streamed(S8KCfg{}, S8KHistCfg{}, kS8K)) != cudaSuccess) return e;
+    if constexpr (FMT == 0) {
+        e = launch_class([&](Launch& LL, int64_t u) { k_step_tile16<4, MODE><<<dim3(u), kThreads, 0, st>>>(LL, P); },
+                         L, pl.idx[kT16V4], t, kT16V4);
+        if (e != cudaSuccess) return e;
+        e = launch_class([&](Launch& LL, int64_t u) { k_step_generic<MODE><<<dim3(u), kThreads, 0, st>>>(LL, P); },
+                         L, pl.idx[kGeneric], t, kGeneric);
+        if (e != cudaSuccess) return e;
+    }
     // Big blocks: partial, finalize, apply per group of tensors.  Chunk and
     // block counters run across groups so workspace slots never collide.
     for (int cls : {kBigAligned, kBigUnaligned}) {
@@ -1467,7 +1575,7 @@ cudaError_t run_step(const Plan& pl, const gefen_tensor_t* t, Launch& L, const P
             }
             L.nunits = units;
             if (units == 0) continue;
-            k_big_partial<MODE><<<dim3(units), kThreads, 0, st>>>(L, P, aligned);
+            k_big_partial<MODE, FMT><<<dim3(units), kThreads, 0, st>>>(L, P, aligned);
             k_big_finalize<MODE><<<dim3(blocks), kThreads, 0, st>>>(L, P);
             if ((e = cudaGetLastError()) != cudaSuccess) return e;
             // apply: streamed tiles where the block size allows, chunks otherwise
@@ -1493,15 +1601,42 @@ cudaError_t run_step(const Plan& pl, const gefen_tensor_t* t, Launch& L, const P
                 }
             }
             if (LS.nunits > 0) {
-                e = (MODE != kPlain && fused) ? stream_kernel<S4KHistCfg, MODE, kFusedBins>(LS, P, err, st)
-                                              : stream_kernel<S4KCfg, MODE, 0>(LS, P, err, st);
+                if constexpr (MODE != kPlain) {
+                    if (fused)
+                        e = stream_kernel<S4KHistCfg, MODE, kFusedBins, FMT>(LS, P, err, st);
+                    else if constexpr (FMT == 0)
+                        e = stream_kernel<S4KCfg, MODE, 0, 0>(LS, P, err, st);
+                    else
+                        e = cudaErrorNotSupported;
+                } else {
+                    e = stream_kernel<S4KCfg, MODE, 0, FMT>(LS, P, err, st);
+                }
                 if (e != cudaSuccess) return e;
             }
-            if (LA.nunits > 0) k_big_apply<MODE><<<dim3(LA.nunits), kThreads, 0, st>>>(LA, P, aligned);
+            if constexpr (FMT == 0) {
+                if (LA.nunits > 0) k_big_apply<MODE><<<dim3(LA.nunits), kThreads, 0, st>>>(LA, P, aligned);
+            } else {
+                if (LA.nunits > 0) return cudaErrorNotSupported;
+            }
             if ((e = cudaGetLastError()) != cudaSuccess) return e;
         }
     }
     return cudaSuccess;
+}
+
+// Whether every tensor's path can store this format: p == 1, the streamed
+// tiles (p a multiple of 32 with two codes per byte) and big blocks applied
+// as streamed tiles.
+bool format_supported(const gefen_tensor_t* t, int32_t n, int fmt) {
+    for (int i = 0; i < n; ++i) {
+        if (t[i].numel == 0) continue;
+        const int64_t p = t[i].period;
+        const PathClass c = classify(p);
+        bool ok = c == kP1 || c == kS4K || c == kS8K || (c == kBigAligned && big_streamable(p));
+        if ((fmt & 1) && (c == kS4K || c == kS8K) && p % 32 != 0) ok = false;
+        if (!ok) return false;
+    }
+    return true;
 }
 
 }  // namespace
@@ -1522,7 +1657,7 @@ extern "C" gefen_status_t gefen_step(const gefen_tensor_t* tensors, int32_t nten
                                      size_t workspace_bytes, gefen_stream_t stream) {
     if (!validate_tensors(tensors, ntensors)) return GEFEN_EINVAL;
     const uint32_t flags = hp.flags;
-    if (flags & ~(GEFEN_HIST | GEFEN_HIST_GRAD_ONLY)) return GEFEN_EINVAL;
+    if (flags & ~(GEFEN_HIST | GEFEN_HIST_GRAD_ONLY | GEFEN_CODES_4BIT | GEFEN_PARAMS_BF16)) return GEFEN_EINVAL;
     if ((flags & GEFEN_HIST) && (flags & GEFEN_HIST_GRAD_ONLY)) return GEFEN_EINVAL;
     const bool grad_only = (flags & GEFEN_HIST_GRAD_ONLY) != 0;
     const bool want_hist = (flags & (GEFEN_HIST | GEFEN_HIST_GRAD_ONLY)) != 0;
@@ -1538,6 +1673,17 @@ extern "C" gefen_status_t gefen_step(const gefen_tensor_t* tensors, int32_t nten
     }
     if (reinterpret_cast<uintptr_t>(grads) & 15u) return GEFEN_EINVAL;
     if (want_hist && (hist == nullptr || hist_bins < 1 || hist_bins > GEFEN_MAX_BINS)) return GEFEN_EINVAL;
+    // storage formats (the first-gradient histogram reads g only)
+    const int fmt = grad_only ? 0 : ((flags & GEFEN_CODES_4BIT) ? 1 : 0) | ((flags & GEFEN_PARAMS_BF16) ? 2 : 0);
+    if (fmt & 1) {
+        if (k > 16) return GEFEN_EINVAL;
+        for (int i = 0; i < ntensors; ++i)
+            if (tensors[i].offset % 32 != 0) return GEFEN_EINVAL;
+    }
+    if (fmt != 0) {
+        if (!format_supported(tensors, ntensors, fmt)) return GEFEN_EUNSUPPORTED;
+        if (want_hist && hist_bins > kFusedBins) return GEFEN_EUNSUPPORTED;
+    }
     const Plan pl = make_plan(tensors, ntensors);
     const WsLayout wl = ws_layout(pl, flags);
     if (workspace_bytes < wl.total || workspace == nullptr) return GEFEN_ENOMEM;
@@ -1579,9 +1725,23 @@ extern "C" gefen_status_t gefen_step(const gefen_tensor_t* tensors, int32_t nten
     cudaError_t e;
     int* err = reinterpret_cast<int*>(ws + wl.header);
     const bool fused = want_hist && hist_bins <= kFusedBins;
-    if (grad_only) e = run_step<kGradOnly>(pl, tensors, L, P, err, st, fused);
-    else if (flags & GEFEN_HIST) e = run_step<kHist>(pl, tensors, L, P, err, st, fused);
-    else e = run_step<kPlain>(pl, tensors, L, P, err, st, false);
+    if (grad_only) {
+        e = run_step<kGradOnly, 0>(pl, tensors, L, P, err, st, fused);
+    } else if (flags & GEFEN_HIST) {
+        switch (fmt) {
+            case 0: e = run_step<kHist, 0>(pl, tensors, L, P, err, st, fused); break;
+            case 1: e = run_step<kHist, 1>(pl, tensors, L, P, err, st, fused); break;
+            case 2: e = run_step<kHist, 2>(pl, tensors, L, P, err, st, fused); break;
+            default: e = run_step<kHist, 3>(pl, tensors, L, P, err, st, fused); break;
+        }
+    } else {
+        switch (fmt) {
+            case 0: e = run_step<kPlain, 0>(pl, tensors, L, P, err, st, false); break;
+            case 1: e = run_step<kPlain, 1>(pl, tensors, L, P, err, st, false); break;
+            case 2: e = run_step<kPlain, 2>(pl, tensors, L, P, err, st, false); break;
+            default: e = run_step<kPlain, 3>(pl, tensors, L, P, err, st, false); break;
+        }
+    }
     if (e != cudaSuccess) return GEFEN_ECUDA;
     if (want_hist) {
         std::vector<HistRange> rr;

@@ -20,6 +20,8 @@ from . import build as _build
 GEFEN_OK, GEFEN_EINVAL, GEFEN_ECUDA, GEFEN_ENOMEM, GEFEN_ETIMEOUT, GEFEN_EUNSUPPORTED, GEFEN_EDEVICE = range(7)
 GEFEN_HIST = 1
 GEFEN_HIST_GRAD_ONLY = 2
+GEFEN_CODES_4BIT = 4
+GEFEN_PARAMS_BF16 = 8
 GEFEN_MAX_BINS = 65536
 GEFEN_MAX_LEVELS = 256
 WS_ALIGN = 256

@@ -96,7 +96,7 @@ def test_step_rejects_bad_scalars_and_pointers():
     assert _step(t, hp=_hp(beta2=-0.1)) == G.GEFEN_EINVAL
     assert _step(t, hp=_hp(eps=float("nan"))) == G.GEFEN_EINVAL
     assert _step(t, hp=_hp(flags=3)) == G.GEFEN_EINVAL
-    assert _step(t, hp=_hp(flags=8)) == G.GEFEN_EINVAL
+    assert _step(t, hp=_hp(flags=16)) == G.GEFEN_EINVAL
     assert _step(t, params=None) == G.GEFEN_EINVAL
     assert _step(t, params=ctypes.c_void_p((1 << 20) + 4)) == G.GEFEN_EINVAL  # misaligned
     assert _step(t, hp=_hp(flags=G.GEFEN_HIST)) == G.GEFEN_EINVAL             # hist missing
@@ -119,3 +119,22 @@ def test_refit_and_infer_reject_bad_arguments():
     assert L.gefen_infer_blocks(P, 64, 0.0, ctypes.byref(per), None, 0, None, P, 1 << 30, None) == G.GEFEN_EINVAL
     assert L.gefen_infer_blocks(P, 64, 1e-8, None, None, 0, None, P, 1 << 30, None) == G.GEFEN_EINVAL
     assert L.gefen_infer_blocks(P, 64, 1e-8, ctypes.byref(per), None, 0, None, P, 8, None) == G.GEFEN_ENOMEM
+
+
+def test_storage_format_checks():
+    t = _table([(0, 64 * 4, 64, 0)])
+    ws = ctypes.c_void_p(1 << 21)
+    # two codes per byte: at most 16 levels, offsets on 32 elements
+    assert _step(t, hp=_hp(flags=G.GEFEN_CODES_4BIT), k=256, ws=ws, ws_bytes=1 << 20) == G.GEFEN_EINVAL
+    assert _step(_table([(16, 64 * 4, 64, 0)]), hp=_hp(flags=G.GEFEN_CODES_4BIT), k=16, ws=ws,
+                 ws_bytes=1 << 20) == G.GEFEN_EINVAL
+    # a shape outside the kernels that store these formats
+    for f in (G.GEFEN_CODES_4BIT, G.GEFEN_PARAMS_BF16):
+        assert _step(_table([(0, 3 * 100, 3, 0)]), hp=_hp(flags=f), k=16, ws=ws, ws_bytes=1 << 20) == \
+            G.GEFEN_EUNSUPPORTED
+    # 4-bit codes need p % 32 == 0 on the streamed tiles
+    assert _step(_table([(0, 48 * 10, 48, 0)]), hp=_hp(flags=G.GEFEN_CODES_4BIT), k=16, ws=ws,
+                 ws_bytes=1 << 20) == G.GEFEN_EUNSUPPORTED
+    # histograms above the in-kernel cells
+    assert _step(t, hp=_hp(flags=G.GEFEN_PARAMS_BF16 | G.GEFEN_HIST), k=16, ws=ws, ws_bytes=1 << 30,
+                 hist=FAKE, bins=8192) == G.GEFEN_EUNSUPPORTED
