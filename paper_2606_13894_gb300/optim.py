@@ -11,8 +11,9 @@ step also histograms the normalised momentum and refits the codebook; the next
 step decodes with the old codebook and encodes with the new one.
 
 All arithmetic of the step runs in the library's CUDA kernels; this module
-only lays out memory and sequences calls.  CUDA fp32 parameters are required:
-there is no CPU path.
+only lays out memory and sequences calls.  CUDA fp32 or bf16 parameters are
+required (bf16 ones are kept in bf16, the update computed in fp32); with at
+most 16 levels the codes are stored two per byte.  There is no CPU path.
 """
 from __future__ import annotations
 
@@ -28,22 +29,25 @@ ALIGN = 64  # elements between tensors in an arena (16 is the library's minimum)
 class _Arena:
     """The packed state of one parameter group."""
 
-    def __init__(self, params: List[torch.nn.Parameter], levels: int, bins: int):
+    def __init__(self, params: List[torch.nn.Parameter], levels: int, bins: int, four_bit: bool):
         dev = params[0].device
+        dtype = params[0].dtype
         self.params = params
+        self.four_bit = four_bit
+        self.flags = (G.GEFEN_CODES_4BIT if four_bit else 0) | (G.GEFEN_PARAMS_BF16 if dtype == torch.bfloat16 else 0)
         self.offsets, o = [], 0
         for p in params:
             self.offsets.append(o)
             o += (p.numel() + ALIGN - 1) // ALIGN * ALIGN
         self.total = max(o, ALIGN)
-        self.theta = torch.zeros(self.total, dtype=torch.float32, device=dev)
+        self.theta = torch.zeros(self.total, dtype=dtype, device=dev)
         with torch.no_grad():
             for p, off in zip(params, self.offsets):
                 self.theta[off:off + p.numel()].copy_(p.detach().reshape(-1))
                 p.data = self.theta[off:off + p.numel()].view_as(p)
         self.grads = torch.zeros(self.total, dtype=torch.bfloat16, device=dev)
         self.gviews = [self.grads[off:off + p.numel()].view_as(p) for p, off in zip(params, self.offsets)]
-        self.codes = torch.zeros(self.total, dtype=torch.uint8, device=dev)
+        self.codes = torch.zeros(self.total // 2 if four_bit else self.total, dtype=torch.uint8, device=dev)
         self.levels, self.bins = levels, bins
         self.cb = torch.empty(levels, dtype=torch.float32, device=dev)
         self.cb_new = torch.empty(levels, dtype=torch.float32, device=dev)
@@ -88,13 +92,18 @@ class Gefen(torch.optim.Optimizer):
     codebook refit (default 16 per level).  refit_every: refit the codebook
     every N steps (0: learn it once, from the first gradient).  periods:
     optional block size of every parameter, all groups in order (default:
-    inferred from the first gradient, Algorithm 2).
+    inferred from the first gradient, Algorithm 2).  four_bit: store the codes
+    two per byte (default: when levels <= 16).  The compact formats (four-bit
+    codes, bf16 parameters) cover blocks of 1, of p <= 8192 with p % 32 == 0
+    (p % 16 == 0 for bf16 alone) and of multiples of 4096; the library
+    reports any other block size as unsupported (give periods= then).
     Parameters without a gradient at a step are left untouched, as in AdamW.
     """
 
     def __init__(self, params, lr: float = 1e-3, betas=(0.9, 0.999), eps: float = 1e-8,
                  weight_decay: float = 1e-2, *, levels: int = 256, bins: Optional[int] = None,
-                 refit_every: int = 0, periods: Optional[Sequence[int]] = None):
+                 refit_every: int = 0, periods: Optional[Sequence[int]] = None,
+                 four_bit: Optional[bool] = None):
         if not 0.0 <= lr or not 0.0 <= eps or not 0.0 <= weight_decay:
             raise ValueError("lr, eps and weight_decay must be non-negative")
         if not (0.0 <= betas[0] < 1.0 and 0.0 <= betas[1] < 1.0):
@@ -108,11 +117,16 @@ class Gefen(torch.optim.Optimizer):
         if not self.levels <= self.bins <= G.GEFEN_MAX_BINS:
             raise ValueError(f"bins must lie in [levels, {G.GEFEN_MAX_BINS}]")
         self.refit_every = int(refit_every)
+        self.four_bit = (self.levels <= 16) if four_bit is None else bool(four_bit)
+        if self.four_bit and self.levels > 16:
+            raise ValueError("four-bit codes hold at most 16 levels")
         self._given_periods = list(periods) if periods is not None else None
         for group in self.param_groups:
             for p in group["params"]:
-                if not p.is_cuda or p.dtype != torch.float32:
-                    raise ValueError("Gefen needs CUDA fp32 parameters (the library has no CPU path)")
+                if not p.is_cuda or p.dtype not in (torch.float32, torch.bfloat16):
+                    raise ValueError("Gefen needs CUDA fp32 or bf16 parameters (the library has no CPU path)")
+            if len({p.dtype for p in group["params"]}) > 1:
+                raise ValueError("the parameters of one group must share a dtype")
         G.load()  # fails loudly when the CUDA library is missing
         self._arenas: List[Optional[_Arena]] = [None] * len(self.param_groups)
         self._pending: Optional[list] = None
@@ -120,7 +134,7 @@ class Gefen(torch.optim.Optimizer):
     # ------------------------------------------------------------ set-up
     def _first_step(self, gi: int, group, present):
         params = list(group["params"])
-        A = _Arena(params, self.levels, self.bins)
+        A = _Arena(params, self.levels, self.bins, self.four_bit)
         self._arenas[gi] = A
         if self._pending is not None and self._pending[gi] is not None:
             self._restore(A, self._pending[gi])
@@ -148,7 +162,8 @@ class Gefen(torch.optim.Optimizer):
                             step=1, flags=G.GEFEN_HIST_GRAD_ONLY, hist=A.hist, workspace_buf=A.ws)
         A.rws = G.gefen_refit_codebook(bins=self.bins, k=self.levels, codebook_out=A.cb, hist_in=A.hist,
                                        workspace_buf=A.rws)
-        A.codes.fill_(int(torch.argmin(A.cb.abs()).item()))  # the level nearest 0, lower index on ties
+        zc = int(torch.argmin(A.cb.abs()).item())  # the level nearest 0, lower index on ties
+        A.codes.fill_(zc | (zc << 4) if A.four_bit else zc)
 
     def _gather(self, A: _Arena, present):
         src = [p.grad for p, ok in zip(A.params, present) if ok]
@@ -181,7 +196,7 @@ class Gefen(torch.optim.Optimizer):
             A.ws = G.gefen_step(A.table_for(present), A.theta, A.grads, A.codes, A.v, A.s, A.cb, enc,
                                 lr=group["lr"], beta1=beta1, beta2=beta2, eps=group["eps"],
                                 weight_decay=group["weight_decay"], step=A.t,
-                                flags=G.GEFEN_HIST if refit else 0, hist=A.hist if refit else None,
+                                flags=A.flags | (G.GEFEN_HIST if refit else 0), hist=A.hist if refit else None,
                                 workspace_buf=A.ws)
             if A.switch:
                 A.cb.copy_(A.cb_new)

@@ -119,3 +119,46 @@ def test_parameters_without_grad_are_untouched():
     assert model[2].weight.grad is None
     opt.step()
     assert torch.equal(model[2].weight, frozen)
+
+
+@pytest.mark.parametrize("dtype,levels", [(torch.float32, 16), (torch.bfloat16, 256), (torch.bfloat16, 16)])
+def test_wrapper_storage_formats_match_the_oracle(dtype, levels):
+    """Four-bit codes (levels <= 16) and bf16 parameters through the wrapper,
+    each step against the oracle (codes unpacked, bf16 widened)."""
+    import test_gpu_formats as F
+    model = _model(5).to(dtype)
+    hp = dict(lr=3e-3, betas=(0.9, 0.99), eps=1e-8, weight_decay=0.05)
+    opt = Gefen(model.parameters(), **hp, levels=levels, refit_every=3)
+    ohp = dict(lr=hp["lr"], beta1=hp["betas"][0], beta2=hp["betas"][1], eps=hp["eps"], weight_decay=hp["weight_decay"])
+    c4 = levels <= 16
+    for i in range(6):
+        x, y = _batch(i)
+        model.zero_grad(set_to_none=True)
+        torch.nn.functional.mse_loss(model(x.to(dtype)).float(), y).backward()
+        A = opt._arenas[0]
+        if A is None:
+            opt.step()
+            continue
+        n = A.total
+        pre = (A.theta.float().cpu().numpy().copy(),
+               F.unpack4(A.codes.cpu().numpy(), n) if c4 else A.codes.cpu().numpy().copy(),
+               A.v.cpu().numpy().copy(), A.s.cpu().numpy().copy())
+        dec = A.cb.cpu().numpy().copy()
+        enc = (A.cb_new if A.switch else A.cb).cpu().numpy().copy()
+        opt.step()
+        gbits = U.bits(A.grads)
+        V = _View(A)
+        th, cd, vv, ss, _ = U.oracle_step(V, pre, gbits, dec, enc, A.t, ohp)
+        got_th = A.theta.float().cpu().numpy()
+        live = np.concatenate([np.arange(o, o + m) for (o, m, _, _) in A.entries])
+        if dtype == torch.bfloat16:
+            ref = th[live].astype(np.float64)
+            tol = 0.5 * F.bf16_ulp(ref) * (1 + 2 ** -10) + U.THETA_TOL * np.maximum(np.abs(ref), ohp["lr"])
+            assert not (np.abs(got_th[live] - ref) > tol).any(), i
+        else:
+            assert U.theta_err(got_th, th, ohp["lr"]) <= U.THETA_TOL, i
+        assert U.rel_err(A.v.cpu().numpy(), vv) <= U.STATE_TOL, i
+        got_cd = F.unpack4(A.codes.cpu().numpy(), n) if c4 else A.codes.cpu().numpy()
+        M = U.summand_scale(V, pre, gbits, dec, ohp["beta1"])
+        assert U.code_flips_ok(V, pre, gbits, dec, enc, got_cd, cd, ohp, M)[0], i
+    opt.check()
