@@ -252,6 +252,50 @@ gefen_status_t gefen_infer_blocks(const uint16_t* grad, int64_t numel, double ep
                                   void* workspace, size_t workspace_bytes,
                                   gefen_stream_t stream);
 
+/* -------------------------------------------------------------------------
+ * gefen_muon_step -- Gefen-Muon (the paper's appendix "Gefen-Muon"): Muon's
+ * momentum buffer kept as Gefen codes with a per-block absmax scale
+ * (Algorithm 1, Quantize), Muon's orthogonalisation unchanged.  For one
+ * rows x cols matrix (row-major), blocks of `period` consecutive elements:
+ *   m    = momentum * codebook_dec[c_i] * s_b + (1 - momentum) * g_i
+ *   s'_b = max |m_i|; c_i = level of codebook_enc nearest m_i / s'_b (ties to
+ *          the lower index; level nearest 0 for s'_b = 0); s_b = s'_b
+ *   U    = g + momentum * (m - g) with nesterov, else m
+ *   X    = U / max(||U||_F, eps), then ns_steps times on the smaller side:
+ *          X <- ns_a X + (ns_b A + ns_c A A) X with A = X X^T
+ *   theta <- theta (1 - lr weight_decay) - lr sqrt(max(1, rows/cols)) X
+ * (Muon as in PyTorch's torch.optim.Muon: momentum 0.95, Nesterov, 5 steps of
+ * (3.4445, -4.7750, 2.0315), eps 1e-7 are its defaults).  The matrix
+ * products run on cuBLAS: fp32, or with GEFEN_MUON_BF16_GEMM bf16 storage and
+ * tensor cores with fp32 accumulation (as Muon runs them).  The first call on
+ * a device creates a cuBLAS handle, which allocates its own small state once;
+ * the products' scratch comes from the workspace.
+ *
+ * params f32[rows*cols], grads bf16[rows*cols] (16-byte aligned), codes
+ * u8[rows*cols], scale f32[rows*cols/period] (device, in/out); codebooks
+ * f32[k] (2 <= k <= 256).  workspace: gefen_muon_workspace_size() bytes,
+ * 256-byte aligned.  rows, cols < 2^31; period divides rows*cols.
+ * ------------------------------------------------------------------------- */
+#define GEFEN_MUON_BF16_GEMM 1u
+
+typedef struct {
+    double lr;
+    double momentum;
+    double weight_decay;
+    double eps;
+    int32_t nesterov;
+    int32_t ns_steps;
+    double ns_a, ns_b, ns_c;
+    uint32_t flags;
+} gefen_muon_hparams_t;
+
+size_t gefen_muon_workspace_size(int64_t rows, int64_t cols, int64_t period, uint32_t flags);
+gefen_status_t gefen_muon_step(int64_t rows, int64_t cols, int64_t period, float* params,
+                               const uint16_t* grads, uint8_t* codes, float* scale,
+                               const float* codebook_dec, const float* codebook_enc, int32_t k,
+                               gefen_muon_hparams_t hp, void* workspace, size_t workspace_bytes,
+                               gefen_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

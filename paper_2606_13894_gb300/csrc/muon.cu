@@ -1,0 +1,298 @@
+// gefen_muon_step: Gefen-Muon (the paper's appendix "Gefen-Muon") on sm_103a.
+//
+// Muon's momentum buffer is kept as Gefen codes with a per-block absmax scale
+// (Algorithm 1, Quantize); the orthogonalisation is Muon's:
+//   m    = mu * Cdec[c] * s_b + (1 - mu) * g           (buffer, decoded + EMA)
+//   s'_b = max |m|, c = nearest level of m / s'_b in Cenc, s_b = s'_b
+//   U    = g + mu (m - g) with Nesterov, else m
+//   X    = U / max(||U||_F, eps); X <- a X + (b A + c A A) X, A = X X^T,
+//          on the smaller side (ns_steps times)
+//   theta = theta (1 - lr wd) - lr sqrt(max(1, rows/cols)) X
+// The element-wise parts are this file's kernels; the Newton-Schulz products
+// are plain GEMMs on cuBLAS (fp32, or bf16 tensor cores like Muon's own).
+//
+// The row-major rows x cols update buffer is, read column-major, the matrix
+// M = X^T (cols x rows).  With rows <= cols the small side is rows: A = M^T M
+// and M <- M B + a M.  With rows > cols it is cols and M is the transposed
+// working matrix itself: A = M M^T and M <- B M + a M.  No transpose is ever
+// materialised.
+#include <cublas_v2.h>
+#include <cuda_bf16.h>
+
+#include <algorithm>
+#include <cmath>
+#include <mutex>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace gefen {
+
+namespace {
+
+constexpr int kMuThreads = 256;
+constexpr int kMuPartials = 1024;  // CTAs of the encode kernel (norm partials)
+constexpr size_t kCublasWs = size_t(32) << 20;
+
+struct MuonLayout {
+    size_t hdr, snew, part, m0, m1, ga, gb, cublas, total;
+};
+
+// header (256 B) | new scales | norm partials | two update buffers | A | B |
+// cuBLAS workspace
+MuonLayout muon_layout(int64_t rows, int64_t cols, int64_t period, bool bf16) {
+    MuonLayout L;
+    const int64_t n = rows * cols, s = std::min(rows, cols);
+    const size_t eb = bf16 ? 2 : 4;
+    size_t o = 0;
+    L.hdr = o; o += kWsAlign;
+    L.snew = o; o += align_up(static_cast<size_t>(n / period) * sizeof(float));
+    L.part = o; o += align_up(static_cast<size_t>(kMuPartials) * sizeof(double));
+    L.m0 = o; o += align_up(static_cast<size_t>(n) * eb);
+    L.m1 = o; o += align_up(static_cast<size_t>(n) * eb);
+    L.ga = o; o += align_up(static_cast<size_t>(s * s) * eb);
+    L.gb = o; o += align_up(static_cast<size_t>(s * s) * eb);
+    L.cublas = o; o += kCublasWs;
+    L.total = o;
+    return L;
+}
+
+struct MuonArgs {
+    int64_t n, period;
+    float mu, omm;  // momentum, 1 - momentum
+    int nesterov, k;
+    const uint16_t* grads;
+    uint8_t* codes;
+    float* scale;
+    const float* cb_dec;
+    const float* cb_enc;
+    float* snew;
+    double* part;
+    void* u;  // update buffer (fp32 or bf16)
+};
+
+__device__ __forceinline__ float muon_m(const MuonArgs& A, const float* s_dec, int64_t e) {
+    const float g = bf16_bits_to_f32(A.grads[e]);
+    return fmaf(A.omm, g, A.mu * A.scale[e / A.period] * s_dec[A.codes[e]]);
+}
+
+// s'_b = max |m| over each block (atomic max of non-negative float bits:
+// exact and order-independent).
+__global__ void __launch_bounds__(kMuThreads) k_muon_absmax(MuonArgs A) {
+    __shared__ float s_dec[kMaxLevels];
+    if (threadIdx.x < kMaxLevels) s_dec[threadIdx.x] = threadIdx.x < A.k ? A.cb_dec[threadIdx.x] : 0.0f;
+    __syncthreads();
+    for (int64_t e = blockIdx.x * static_cast<int64_t>(kMuThreads) + threadIdx.x; e < A.n;
+         e += static_cast<int64_t>(gridDim.x) * kMuThreads) {
+        const float am = fabsf(muon_m(A, s_dec, e));
+        atomicMax(reinterpret_cast<unsigned int*>(A.snew) + e / A.period, __float_as_uint(am));
+    }
+}
+
+// Re-encode, write the update U and each CTA's partial sum of U^2.
+template <bool BF16>
+__global__ void __launch_bounds__(kMuThreads) k_muon_encode(MuonArgs A) {
+    __shared__ float s_dec[kMaxLevels], s_mid[kMaxLevels];
+    __shared__ double s_red[kMuThreads / 32];
+    const int t = threadIdx.x;
+    if (t < kMaxLevels) {
+        s_dec[t] = t < A.k ? A.cb_dec[t] : 0.0f;
+        s_mid[t] = (t < A.k - 1) ? 0.5f * (A.cb_enc[t] + A.cb_enc[t + 1]) : INFINITY;
+    }
+    __syncthreads();
+    const int zero_code = level_search(s_mid, 0.0f);
+    double acc = 0.0;
+    for (int64_t e = blockIdx.x * static_cast<int64_t>(kMuThreads) + t; e < A.n;
+         e += static_cast<int64_t>(gridDim.x) * kMuThreads) {
+        const float g = bf16_bits_to_f32(A.grads[e]);
+        const float m = fmaf(A.omm, g, A.mu * A.scale[e / A.period] * s_dec[A.codes[e]]);
+        const float sn = A.snew[e / A.period];
+        A.codes[e] = static_cast<uint8_t>(sn > 0.0f ? level_search(s_mid, __fdiv_rn(m, sn)) : zero_code);
+        const float u = A.nesterov ? fmaf(A.mu, m - g, g) : m;
+        if (BF16) {
+            const __nv_bfloat16 ub = __float2bfloat16_rn(u);
+            reinterpret_cast<__nv_bfloat16*>(A.u)[e] = ub;
+            const double ud = static_cast<double>(__bfloat162float(ub));
+            acc += ud * ud;
+        } else {
+            reinterpret_cast<float*>(A.u)[e] = u;
+            acc += static_cast<double>(u) * u;
+        }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if ((t & 31) == 0) s_red[t >> 5] = acc;
+    __syncthreads();
+    if (t == 0) {
+        double s = 0.0;
+        for (int w = 0; w < kMuThreads / 32; ++w) s += s_red[w];
+        A.part[blockIdx.x] = s;
+    }
+}
+
+// Normalise U (one fixed-order sum of the partials) and commit the new scales.
+template <bool BF16>
+__global__ void __launch_bounds__(kMuThreads) k_muon_normalise(MuonArgs A, int nparts, double eps) {
+    __shared__ float s_inv;
+    if (threadIdx.x == 0) {
+        double s = 0.0;
+        for (int i = 0; i < nparts; ++i) s += A.part[i];
+        s_inv = static_cast<float>(1.0 / fmax(sqrt(s), eps));
+    }
+    __syncthreads();
+    const float inv = s_inv;
+    const int64_t nb = A.n / A.period;
+    for (int64_t e = blockIdx.x * static_cast<int64_t>(kMuThreads) + threadIdx.x; e < A.n;
+         e += static_cast<int64_t>(gridDim.x) * kMuThreads) {
+        if (BF16) {
+            __nv_bfloat16* u = reinterpret_cast<__nv_bfloat16*>(A.u);
+            u[e] = __float2bfloat16_rn(__bfloat162float(u[e]) * inv);
+        } else {
+            float* u = reinterpret_cast<float*>(A.u);
+            u[e] *= inv;
+        }
+        if (e < nb) A.scale[e] = A.snew[e];
+    }
+}
+
+template <bool BF16>
+__global__ void __launch_bounds__(kMuThreads) k_muon_update(float* __restrict__ theta, const void* __restrict__ x,
+                                                         int64_t n, float decay, float step) {
+    for (int64_t e = blockIdx.x * static_cast<int64_t>(kMuThreads) + threadIdx.x; e < n;
+         e += static_cast<int64_t>(gridDim.x) * kMuThreads) {
+        const float xv = BF16 ? __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(x)[e])
+                              : reinterpret_cast<const float*>(x)[e];
+        theta[e] = fmaf(-step, xv, decay * theta[e]);
+    }
+}
+
+// One cuBLAS handle per device, created on first use (cuBLAS keeps its own
+// state; its scratch for our calls comes from the caller's workspace).
+cublasHandle_t muon_handle() {
+    static std::mutex mu;
+    static cublasHandle_t h[64] = {nullptr};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    std::lock_guard<std::mutex> g(mu);
+    if (!h[dev] && cublasCreate(&h[dev]) != CUBLAS_STATUS_SUCCESS) h[dev] = nullptr;
+    return h[dev];
+}
+
+// C = alpha op(A) op(B) + beta C, column-major, fp32 or bf16 storage with fp32
+// accumulation.
+cublasStatus_t gemm(cublasHandle_t h, bool bf16, cublasOperation_t ta, cublasOperation_t tb, int m, int n, int k,
+                    float alpha, const void* A, int lda, const void* B, int ldb, float beta, void* C, int ldc) {
+    const cudaDataType_t ty = bf16 ? CUDA_R_16BF : CUDA_R_32F;
+    return cublasGemmEx(h, ta, tb, m, n, k, &alpha, A, ty, lda, B, ty, ldb, &beta, C, ty, ldc,
+                        CUBLAS_COMPUTE_32F, CUBLAS_GEMM_DEFAULT);
+}
+
+}  // namespace
+
+}  // namespace gefen
+
+using namespace gefen;
+
+extern "C" size_t gefen_muon_workspace_size(int64_t rows, int64_t cols, int64_t period, uint32_t flags) {
+    if (rows < 1 || cols < 1 || period < 1 || (rows * cols) % period != 0) return 0;
+    if (rows > (int64_t(1) << 31) - 1 || cols > (int64_t(1) << 31) - 1) return 0;
+    return muon_layout(rows, cols, period, (flags & GEFEN_MUON_BF16_GEMM) != 0).total;
+}
+
+extern "C" gefen_status_t gefen_muon_step(int64_t rows, int64_t cols, int64_t period, float* params,
+                                          const uint16_t* grads, uint8_t* codes, float* scale,
+                                          const float* codebook_dec, const float* codebook_enc, int32_t k,
+                                          gefen_muon_hparams_t hp, void* workspace, size_t workspace_bytes,
+                                          gefen_stream_t stream) {
+    if (rows < 1 || cols < 1 || period < 1 || (rows * cols) % period != 0) return GEFEN_EINVAL;
+    if (rows > (int64_t(1) << 31) - 1 || cols > (int64_t(1) << 31) - 1) return GEFEN_EINVAL;
+    if (!params || !grads || !codes || !scale || !codebook_dec || !codebook_enc) return GEFEN_EINVAL;
+    if (k < 2 || k > GEFEN_MAX_LEVELS) return GEFEN_EINVAL;
+    if (hp.flags & ~GEFEN_MUON_BF16_GEMM) return GEFEN_EINVAL;
+    if (!(hp.momentum >= 0.0 && hp.momentum < 1.0) || !std::isfinite(hp.lr) || !std::isfinite(hp.weight_decay) ||
+        !(hp.eps > 0.0) || hp.ns_steps < 0 || hp.ns_steps > 100 || !std::isfinite(hp.ns_a) ||
+        !std::isfinite(hp.ns_b) || !std::isfinite(hp.ns_c))
+        return GEFEN_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(params) | reinterpret_cast<uintptr_t>(grads)) & 15u) return GEFEN_EINVAL;
+    const bool bf16 = (hp.flags & GEFEN_MUON_BF16_GEMM) != 0;
+    const MuonLayout L = muon_layout(rows, cols, period, bf16);
+    if (workspace == nullptr || workspace_bytes < L.total) return GEFEN_ENOMEM;
+    if (reinterpret_cast<uintptr_t>(workspace) % kWsAlign) return GEFEN_EINVAL;
+    if (gefen_status_t s = check_device(); s != GEFEN_OK) return s;
+    cublasHandle_t h = muon_handle();
+    if (!h) return GEFEN_ECUDA;
+
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    char* ws = static_cast<char*>(workspace);
+    const int64_t n = rows * cols;
+    MuonArgs A;
+    A.n = n;
+    A.period = period;
+    A.mu = static_cast<float>(hp.momentum);
+    A.omm = static_cast<float>(1.0 - hp.momentum);
+    A.nesterov = hp.nesterov ? 1 : 0;
+    A.k = k;
+    A.grads = grads;
+    A.codes = codes;
+    A.scale = scale;
+    A.cb_dec = codebook_dec;
+    A.cb_enc = codebook_enc;
+    A.snew = reinterpret_cast<float*>(ws + L.snew);
+    A.part = reinterpret_cast<double*>(ws + L.part);
+    void* M = ws + L.m0;
+    void* Mn = ws + L.m1;
+    void* GA = ws + L.ga;
+    void* GB = ws + L.gb;
+    A.u = M;
+
+    const int grid = static_cast<int>(std::min<int64_t>(kMuPartials, (n + kMuThreads - 1) / kMuThreads));
+    if (cudaMemsetAsync(A.snew, 0, static_cast<size_t>(n / period) * sizeof(float), st) != cudaSuccess)
+        return GEFEN_ECUDA;
+    k_muon_absmax<<<grid, kMuThreads, 0, st>>>(A);
+    if (bf16) {
+        k_muon_encode<true><<<grid, kMuThreads, 0, st>>>(A);
+        k_muon_normalise<true><<<grid, kMuThreads, 0, st>>>(A, grid, hp.eps);
+    } else {
+        k_muon_encode<false><<<grid, kMuThreads, 0, st>>>(A);
+        k_muon_normalise<false><<<grid, kMuThreads, 0, st>>>(A, grid, hp.eps);
+    }
+    if (cudaGetLastError() != cudaSuccess) return GEFEN_ECUDA;
+
+    // Newton-Schulz on the column-major view M (cols x rows, ld = cols)
+    if (cublasSetStream(h, st) != CUBLAS_STATUS_SUCCESS ||
+        cublasSetWorkspace(h, ws + L.cublas, kCublasWs) != CUBLAS_STATUS_SUCCESS ||
+        cublasSetMathMode(h, CUBLAS_DEFAULT_MATH) != CUBLAS_STATUS_SUCCESS)
+        return GEFEN_ECUDA;
+    const bool wide = rows <= cols;
+    const int s = static_cast<int>(std::min(rows, cols));
+    const int ld = static_cast<int>(cols), nr = static_cast<int>(rows);
+    const size_t eb = bf16 ? 2 : 4;
+    const float a = static_cast<float>(hp.ns_a), b = static_cast<float>(hp.ns_b), c = static_cast<float>(hp.ns_c);
+    for (int it = 0; it < hp.ns_steps; ++it) {
+        cublasStatus_t cs;
+        // A = X X^T on the small side
+        cs = wide ? gemm(h, bf16, CUBLAS_OP_T, CUBLAS_OP_N, s, s, ld, 1.0f, M, ld, M, ld, 0.0f, GA, s)
+                  : gemm(h, bf16, CUBLAS_OP_N, CUBLAS_OP_T, s, s, nr, 1.0f, M, ld, M, ld, 0.0f, GA, s);
+        if (cs != CUBLAS_STATUS_SUCCESS) return GEFEN_ECUDA;
+        // B = b A + c A A
+        if (cudaMemcpyAsync(GB, GA, static_cast<size_t>(s) * s * eb, cudaMemcpyDeviceToDevice, st) != cudaSuccess)
+            return GEFEN_ECUDA;
+        if (gemm(h, bf16, CUBLAS_OP_N, CUBLAS_OP_N, s, s, s, c, GA, s, GA, s, b, GB, s) != CUBLAS_STATUS_SUCCESS)
+            return GEFEN_ECUDA;
+        // X <- a X + B X  (M <- M B + a M, or M <- B M + a M)
+        if (cudaMemcpyAsync(Mn, M, static_cast<size_t>(n) * eb, cudaMemcpyDeviceToDevice, st) != cudaSuccess)
+            return GEFEN_ECUDA;
+        cs = wide ? gemm(h, bf16, CUBLAS_OP_N, CUBLAS_OP_N, ld, s, s, 1.0f, M, ld, GB, s, a, Mn, ld)
+                  : gemm(h, bf16, CUBLAS_OP_N, CUBLAS_OP_N, s, nr, s, 1.0f, GB, s, M, ld, a, Mn, ld);
+        if (cs != CUBLAS_STATUS_SUCCESS) return GEFEN_ECUDA;
+        std::swap(M, Mn);
+    }
+    const double adj = hp.lr * std::sqrt(std::max(1.0, static_cast<double>(rows) / static_cast<double>(cols)));
+    const float decay = static_cast<float>(1.0 - hp.lr * hp.weight_decay);
+    if (bf16)
+        k_muon_update<true><<<grid, kMuThreads, 0, st>>>(params, M, n, decay, static_cast<float>(adj));
+    else
+        k_muon_update<false><<<grid, kMuThreads, 0, st>>>(params, M, n, decay, static_cast<float>(adj));
+    if (cudaGetLastError() != cudaSuccess) return GEFEN_ECUDA;
+    return GEFEN_OK;
+}

@@ -48,7 +48,16 @@ EXPORTS = ("gefen_status_string", "gefen_sync_status", "gefen_step_workspace_siz
            "gefen_step_status",
            "gefen_refit_workspace_size", "gefen_refit_codebook", "gefen_refit_status",
            "gefen_refit_tables", "gefen_infer_workspace_size", "gefen_infer_blocks",
-           "gefen_refit_codebook_static")
+           "gefen_refit_codebook_static", "gefen_muon_workspace_size", "gefen_muon_step")
+
+GEFEN_MUON_BF16_GEMM = 1
+
+
+class gefen_muon_hparams_t(ctypes.Structure):
+    _fields_ = [("lr", ctypes.c_double), ("momentum", ctypes.c_double), ("weight_decay", ctypes.c_double),
+                ("eps", ctypes.c_double), ("nesterov", ctypes.c_int32), ("ns_steps", ctypes.c_int32),
+                ("ns_a", ctypes.c_double), ("ns_b", ctypes.c_double), ("ns_c", ctypes.c_double),
+                ("flags", ctypes.c_uint32)]
 
 _lib = None
 _lock = threading.Lock()
@@ -96,6 +105,10 @@ def load(build_if_needed: bool = True):
                                          ctypes.POINTER(ctypes.c_double), i64, ctypes.POINTER(i64),
                                          P, sz, P]
         L.gefen_infer_blocks.restype = ctypes.c_int
+        L.gefen_muon_workspace_size.argtypes = [i64, i64, i64, ctypes.c_uint32]
+        L.gefen_muon_workspace_size.restype = sz
+        L.gefen_muon_step.argtypes = [i64, i64, i64, P, P, P, P, P, P, i32, gefen_muon_hparams_t, P, sz, P]
+        L.gefen_muon_step.restype = ctypes.c_int
         _lib = L
         return L
 
@@ -256,3 +269,27 @@ def gefen_infer_blocks(grad, eps: float = 1e-8, *, workspace_buf=None, want_scor
                                    _ptr(workspace_buf), workspace_buf.numel(), _stream(stream))
     _check("gefen_infer_blocks", st)
     return int(period.value), [scores[i] for i in range(min(cap, nd.value))]
+
+
+MUON_NS = (3.4445, -4.7750, 2.0315)
+
+
+def gefen_muon_workspace_size(rows: int, cols: int, period: int, flags: int = 0) -> int:
+    return int(load().gefen_muon_workspace_size(rows, cols, period, flags))
+
+
+def gefen_muon_step(rows, cols, period, params, grads, codes, scale, codebook_dec, codebook_enc, *, lr,
+                    momentum=0.95, weight_decay=0.1, eps=1e-7, nesterov=True, ns_steps=5, ns=MUON_NS,
+                    flags=0, workspace_buf=None, stream=None):
+    """One Gefen-Muon step on a rows x cols matrix (see gefen.h).  Returns the
+    workspace used."""
+    need = gefen_muon_workspace_size(rows, cols, period, flags)
+    if workspace_buf is None or workspace_buf.numel() < need:
+        workspace_buf = workspace(need, params.device)
+    hp = gefen_muon_hparams_t(float(lr), float(momentum), float(weight_decay), float(eps), int(bool(nesterov)),
+                              int(ns_steps), float(ns[0]), float(ns[1]), float(ns[2]), int(flags))
+    st = load().gefen_muon_step(rows, cols, period, _ptr(params), _ptr(grads), _ptr(codes), _ptr(scale),
+                                _ptr(codebook_dec), _ptr(codebook_enc), codebook_enc.numel(), hp,
+                                _ptr(workspace_buf), workspace_buf.numel(), _stream(stream))
+    _check("gefen_muon_step", st)
+    return workspace_buf

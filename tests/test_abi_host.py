@@ -138,3 +138,20 @@ def test_storage_format_checks():
     # histograms above the in-kernel cells
     assert _step(t, hp=_hp(flags=G.GEFEN_PARAMS_BF16 | G.GEFEN_HIST), k=16, ws=ws, ws_bytes=1 << 30,
                  hist=FAKE, bins=8192) == G.GEFEN_EUNSUPPORTED
+
+
+def test_muon_rejects_bad_arguments():
+    L = G.load()
+    hp = G.gefen_muon_hparams_t(1e-3, 0.95, 0.1, 1e-7, 1, 5, 3.4445, -4.775, 2.0315, 0)
+    P = FAKE
+    big = 1 << 30
+    assert L.gefen_muon_step(0, 8, 1, P, P, P, P, P, P, 16, hp, P, big, None) == G.GEFEN_EINVAL
+    assert L.gefen_muon_step(4, 8, 3, P, P, P, P, P, P, 16, hp, P, big, None) == G.GEFEN_EINVAL  # 3 does not divide 32
+    assert L.gefen_muon_step(4, 8, 8, P, P, P, P, P, P, 1, hp, P, big, None) == G.GEFEN_EINVAL
+    bad = G.gefen_muon_hparams_t(1e-3, 1.0, 0.1, 1e-7, 1, 5, 3.4445, -4.775, 2.0315, 0)
+    assert L.gefen_muon_step(4, 8, 8, P, P, P, P, P, P, 16, bad, P, big, None) == G.GEFEN_EINVAL
+    badf = G.gefen_muon_hparams_t(1e-3, 0.9, 0.1, 1e-7, 1, 5, 3.4445, -4.775, 2.0315, 4)
+    assert L.gefen_muon_step(4, 8, 8, P, P, P, P, P, P, 16, badf, P, big, None) == G.GEFEN_EINVAL
+    assert L.gefen_muon_step(4, 8, 8, P, P, P, P, P, P, 16, hp, P, 64, None) == G.GEFEN_ENOMEM
+    assert G.gefen_muon_workspace_size(4, 8, 3) == 0
+    assert G.gefen_muon_workspace_size(64, 256, 64) > 2 * 64 * 256 * 4
