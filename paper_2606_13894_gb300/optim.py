@@ -254,3 +254,106 @@ class Gefen(torch.optim.Optimizer):
             if src.numel() != dst.numel():
                 raise ValueError(f"checkpoint {name} has {src.numel()} entries, expected {dst.numel()}")
             dst.copy_(src.to(dst.device))
+
+
+class GefenMuon(torch.optim.Optimizer):
+    """Gefen-Muon (the paper's appendix "Gefen-Muon") with Muon's arguments:
+    Muon's momentum buffer kept as Gefen codes and per-block scales, Muon's
+    orthogonalisation (gefen_muon_step).  Like Muon it is for matrices: a
+    parameter of more than two dimensions is viewed as (dim 0, the rest); a
+    vector is refused.  Blocks are inferred per matrix from its first
+    gradient (Algorithm 2) unless periods are given; the codebook is learned
+    once from the first gradients (Algorithm 3).  bf16_products runs the
+    Newton-Schulz products on bf16 tensor cores, as Muon does.
+    """
+
+    def __init__(self, params, lr: float = 1e-3, weight_decay: float = 0.1, momentum: float = 0.95,
+                 nesterov: bool = True, ns_coefficients=G.MUON_NS, eps: float = 1e-7, ns_steps: int = 5, *,
+                 levels: int = 256, bins: Optional[int] = None, periods: Optional[Sequence[int]] = None,
+                 bf16_products: bool = True):
+        if not 0.0 <= momentum < 1.0:
+            raise ValueError("momentum must lie in [0, 1)")
+        defaults = dict(lr=lr, weight_decay=weight_decay, momentum=momentum, nesterov=nesterov,
+                        ns_coefficients=tuple(ns_coefficients), eps=eps, ns_steps=ns_steps)
+        super().__init__(params, defaults)
+        self.levels = int(levels)
+        self.bins = int(bins) if bins else 16 * self.levels
+        self.flags = G.GEFEN_MUON_BF16_GEMM if bf16_products else 0
+        self._given_periods = list(periods) if periods is not None else None
+        for group in self.param_groups:
+            for p in group["params"]:
+                if not p.is_cuda or p.dtype != torch.float32 or p.dim() < 2 or not p.is_contiguous():
+                    raise ValueError("GefenMuon needs contiguous CUDA fp32 matrices (the library has no CPU path)")
+        G.load()
+        self._setup = [None] * len(self.param_groups)
+        self._ws = None
+
+    @staticmethod
+    def _shape(p):
+        return p.shape[0], p.numel() // p.shape[0]
+
+    def _first_step(self, gi, group):
+        params = [p for p in group["params"]]
+        if any(p.grad is None for p in params):
+            raise RuntimeError("the first step needs a gradient for every parameter (it learns the codebook)")
+        dev = params[0].device
+        offs, o = [], 0
+        for p in params:
+            offs.append(o)
+            o += (p.numel() + 63) // 64 * 64
+        garena = torch.zeros(max(o, 64), dtype=torch.bfloat16, device=dev)
+        for p, off in zip(params, offs):
+            garena[off:off + p.numel()].copy_(p.grad.reshape(-1))
+        if self._given_periods is not None:
+            start = sum(len(g["params"]) for g in self.param_groups[:gi])
+            periods = self._given_periods[start:start + len(params)]
+        else:
+            periods, iws = [], None
+            for p, off in zip(params, offs):
+                need = G.gefen_infer_workspace_size(p.numel())
+                if iws is None or iws.numel() < need:
+                    iws = G.workspace(need, dev)
+                per, _ = G.gefen_infer_blocks(garena[off:off + p.numel()], 1e-8, workspace_buf=iws,
+                                              want_scores=False)
+                periods.append(per)
+        entries, b = [], 0
+        for p, off, per in zip(params, offs, periods):
+            entries.append((off, p.numel(), per, b))
+            b += p.numel() // per
+        table = G.tensor_table(entries)
+        hist = torch.zeros(self.bins, dtype=torch.int64, device=dev)
+        cb = torch.empty(self.levels, dtype=torch.float32, device=dev)
+        dummy = torch.zeros(max(b, 1), dtype=torch.float32, device=dev)
+        G.gefen_step(table, None, garena, None, dummy, dummy, cb, cb, lr=0.0, beta1=0.0, beta2=0.0, eps=1.0,
+                     weight_decay=0.0, step=1, flags=G.GEFEN_HIST_GRAD_ONLY, hist=hist)
+        G.gefen_refit_codebook(bins=self.bins, k=self.levels, codebook_out=cb, hist_in=hist)
+        zc = int(torch.argmin(cb.abs()).item())
+        states = []
+        for p, per in zip(params, periods):
+            states.append(dict(period=int(per), codes=torch.full((p.numel(),), zc, dtype=torch.uint8, device=dev),
+                               scale=torch.zeros(p.numel() // per, dtype=torch.float32, device=dev)))
+        self._setup[gi] = dict(cb=cb, states=states)
+
+    @torch.no_grad()
+    def step(self, closure=None):
+        loss = None
+        if closure is not None:
+            with torch.enable_grad():
+                loss = closure()
+        for gi, group in enumerate(self.param_groups):
+            if self._setup[gi] is None:
+                if all(p.grad is None for p in group["params"]):
+                    continue
+                self._first_step(gi, group)
+            S = self._setup[gi]
+            for p, st in zip(group["params"], S["states"]):
+                if p.grad is None:
+                    continue
+                rows, cols = self._shape(p)
+                g = p.grad.reshape(-1).to(torch.bfloat16).contiguous()
+                self._ws = G.gefen_muon_step(rows, cols, st["period"], p.data, g, st["codes"], st["scale"],
+                                             S["cb"], S["cb"], lr=group["lr"], momentum=group["momentum"],
+                                             weight_decay=group["weight_decay"], eps=group["eps"],
+                                             nesterov=group["nesterov"], ns_steps=group["ns_steps"],
+                                             ns=group["ns_coefficients"], flags=self.flags, workspace_buf=self._ws)
+        return loss

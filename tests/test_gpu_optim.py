@@ -162,3 +162,44 @@ def test_wrapper_storage_formats_match_the_oracle(dtype, levels):
         M = U.summand_scale(V, pre, gbits, dec, ohp["beta1"])
         assert U.code_flips_ok(V, pre, gbits, dec, enc, got_cd, cd, ohp, M)[0], i
     opt.check()
+
+
+@pytest.mark.parametrize("bf16_products", [False, True])
+def test_gefen_muon_wrapper_steps_match_the_oracle(bf16_products):
+    """GefenMuon on the matrices of a small MLP: every step against the
+    Gefen-Muon oracle from the wrapper's own pre-step state."""
+    import math
+    from oracle import muon as OM
+    from paper_2606_13894_gb300.optim import GefenMuon
+    torch.manual_seed(6)
+    model = torch.nn.Sequential(torch.nn.Linear(64, 256, bias=False), torch.nn.ReLU(),
+                                torch.nn.Linear(256, 32, bias=False)).cuda()
+    hp = dict(lr=2e-2, weight_decay=0.1, momentum=0.9)
+    opt = GefenMuon(model.parameters(), **hp, bf16_products=bf16_products)
+    tolx = 6e-2 if bf16_products else 2e-4
+    for i in range(5):
+        _backward(model, i)
+        if opt._setup[0] is None:
+            opt.step()
+            continue
+        S = opt._setup[0]
+        cb = S["cb"].cpu().numpy()
+        pres = []
+        for p, st in zip(model.parameters(), S["states"]):
+            pres.append((p.detach().reshape(-1).cpu().numpy().copy(), st["codes"].cpu().numpy().copy(),
+                         st["scale"].cpu().numpy().copy(), U.bits(p.grad.reshape(-1).to(torch.bfloat16))))
+        opt.step()
+        for (th0, cd0, s0, gbits), p, st in zip(pres, model.parameters(), S["states"]):
+            rows, cols = p.shape[0], p.numel() // p.shape[0]
+            th, cd, ss = th0.copy(), cd0.copy(), s0.copy()
+            X = OM.muon_step(th, gbits, cd, ss, cb, cb, rows=rows, cols=cols, period=st["period"], **hp)
+            adj = hp["lr"] * math.sqrt(max(1.0, rows / cols))
+            tol = adj * tolx * np.abs(X).max() + 1e-5 * np.maximum(np.abs(th.astype(np.float64)), hp["lr"])
+            got = p.detach().reshape(-1).cpu().numpy().astype(np.float64)
+            assert np.all(np.abs(got - th) <= tol), i
+            V = _View(type("A", (), {"entries": [(0, p.numel(), st["period"], 0)], "v": st["scale"]})())
+            pre = (th0, cd0, np.zeros(1, np.float32), s0)
+            Mb = U.summand_scale(V, pre, gbits, cb, hp["momentum"])
+            assert U.scale_ok(st["scale"].cpu().numpy(), ss, Mb)[0], i
+            assert U.code_flips_ok(V, pre, gbits, cb, cb, st["codes"].cpu().numpy(), cd,
+                                   dict(beta1=hp["momentum"]), Mb)[0], i
