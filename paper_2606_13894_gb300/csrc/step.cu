@@ -689,6 +689,31 @@ __device__ __forceinline__ void butterfly(float& s2, float& mx, int lanes) {
     }
 }
 
+// Warp maxima and sums for block reductions.  A maximum of magnitudes (>= 0,
+// never NaN: fmaxf drops NaN) is one integer max over the float bits, which
+// order like the values; a sum is a five-level butterfly.
+__device__ __forceinline__ float warp_max_nonneg(float x) {
+    return __uint_as_float(__reduce_max_sync(0xffffffffu, __float_as_uint(x)));
+}
+__device__ __forceinline__ float warp_sum_bfly(float x) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+    return x;
+}
+// Hardware approximations (about 1 ulp): the step factor and the scale's
+// reciprocal feed the parameter update and the nearest-level decision, both
+// far inside the 1e-5 parameter and 1e-6 decision-margin tolerances.
+__device__ __forceinline__ float rcp_approx(float x) {
+    float r;
+    asm("rcp.approx.f32 %0, %1;" : "=f"(r) : "f"(x));
+    return r;
+}
+__device__ __forceinline__ float sqrt_approx(float x) {
+    float r;
+    asm("sqrt.approx.f32 %0, %1;" : "=f"(r) : "f"(x));
+    return r;
+}
+
 // 0xFFFFFFFF if a < b else 0 (one compare that yields an integer mask)
 __device__ __forceinline__ uint32_t lt_mask(float a, float b) {
     uint32_t r;
@@ -725,7 +750,8 @@ __device__ __forceinline__ void encode4(const StreamTables<LUTR, DECR>& T, int c
 // tile holds TILE elements), so no group needs a bounds predicate.
 template <int TILE, int THREADS, int LUTR, int DECR, int MODE, bool THS, int FMT, bool LUT, bool FULL, typename Smem>
 __device__ __forceinline__ void stream_tile(Smem& sm, const Ptrs& P, const HP& hp, const TileInfo& ti,
-                                            unsigned char* st, int eb, const float (&r_s)[4], const float (&r_v)[4]) {
+                                            unsigned char* st, int eb, const float (&r_s)[4], const float (&r_v)[4],
+                                            const float4 (&th)[4]) {
     using SL = StageLayout<TILE, THS, FMT>;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int lut_copy = lane % LUTR, dec_copy = lane % DECR;
@@ -740,12 +766,6 @@ __device__ __forceinline__ void stream_tile(Smem& sm, const Ptrs& P, const HP& h
         blk[j] = static_cast<int>(__umulhi(static_cast<uint32_t>(e), ti.pmagic));
     }
     const int64_t ge0 = ti.e0 + eb;  // element of group 0; group j at + 128 j
-    float4 th[4];  // theta from global memory is loaded early; from the stage, just before use
-    if (MODE != kGradOnly && !THS) {
-#pragma unroll
-        for (int j = 0; j < 4; ++j)
-            if (live[j]) th[j] = theta4_global<FMT>(P.params, ge0 + 128 * j);
-    }
 
     // phase 1: decode m, partials per group of four
     float m[16], g2[4], mx[4];
@@ -787,8 +807,8 @@ __device__ __forceinline__ void stream_tile(Smem& sm, const Ptrs& P, const HP& h
             f = 0.0f;
         } else {
             const float vn = fmaf(hp.beta2, v_old, hp.omb2 * (s2 * rp));
-            f = hp.lr_bc1 * __frcp_rn(sqrtf(vn * hp.inv_bc2) + hp.eps);
-            iv = sx > 0.0f ? __frcp_rn(sx) : 0.0f;
+            f = hp.lr_bc1 * rcp_approx(sqrt_approx(vn * hp.inv_bc2) + hp.eps);
+            iv = sx > 0.0f ? rcp_approx(sx) : 0.0f;
             if (writer) {
                 P.v[bi] = vn;
                 P.scale[bi] = sx;
@@ -803,9 +823,8 @@ __device__ __forceinline__ void stream_tile(Smem& sm, const Ptrs& P, const HP& h
         for (int j = 0; j < 4; ++j) { fac[j] = bs.z; inv[j] = iv; }
     } else if ((p & 511) == 0) {
         // a warp's 512 elements lie in one block
-        float s2 = (g2[0] + g2[1]) + (g2[2] + g2[3]);
-        float sx = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
-        butterfly(s2, sx, 32);
+        float s2 = warp_sum_bfly((g2[0] + g2[1]) + (g2[2] + g2[3]));
+        float sx = warp_max_nonneg(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])));
         const int nw = p >> 9;  // warps per block
         if (nw > 1) {
             if (lane == 0) sm.part[warp] = make_float2(s2, sx);
@@ -824,10 +843,8 @@ __device__ __forceinline__ void stream_tile(Smem& sm, const Ptrs& P, const HP& h
         for (int j = 1; j < 4; ++j) { fac[j] = fac[0]; inv[j] = inv[0]; }
     } else if (p == 256) {
         // groups 0,1 and 2,3 form one block each
-        float s0 = g2[0] + g2[1], x0 = fmaxf(mx[0], mx[1]);
-        float s1 = g2[2] + g2[3], x1 = fmaxf(mx[2], mx[3]);
-        butterfly(s0, x0, 32);
-        butterfly(s1, x1, 32);
+        const float s0 = warp_sum_bfly(g2[0] + g2[1]), x0 = warp_max_nonneg(fmaxf(mx[0], mx[1]));
+        const float s1 = warp_sum_bfly(g2[2] + g2[3]), x1 = warp_max_nonneg(fmaxf(mx[2], mx[3]));
         finish(s0, x0, r_v[0], ti.bo + blk[0], live[0] && lane == 0, fac[0], inv[0]);
         finish(s1, x1, r_v[2], ti.bo + blk[2], live[2] && lane == 0, fac[2], inv[2]);
         fac[1] = fac[0]; inv[1] = inv[0];
@@ -947,6 +964,15 @@ __device__ __forceinline__ void stream_loop(Smem& sm, const Launch& L, const Ptr
             if (tid == 0) atomicExch(err, 2);
             break;
         }
+        // theta from global memory (an L2 hit: prefetched when the tile was
+        // issued) is requested before the stage wait; from the stage, just
+        // before use
+        float4 th[4];
+        if (MODE != kGradOnly && !THS) {
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+                if (eb + 128 * j < ti.nelem) th[j] = theta4_global<FMT>(P.params, ti.e0 + eb + 128 * j);
+        }
         // each thread waits for the stage itself; a wait that gives up is
         // acted on, uniformly, at the end of the tile
         const bool ok = mbar_wait(smem_u32(&sm.bar[s]), parity);
@@ -957,9 +983,9 @@ __device__ __forceinline__ void stream_loop(Smem& sm, const Launch& L, const Ptr
             load_state<4>(P, sm.tile[(it + 1) % STAGES], eb, n_s, n_v);
 
         if (ti.nelem == TILE)
-            stream_tile<TILE, THREADS, LUTR, DECR, MODE, THS, FMT, LUT, true>(sm, P, L.hp, ti, sm.stage[s], eb, r_s, r_v);
+            stream_tile<TILE, THREADS, LUTR, DECR, MODE, THS, FMT, LUT, true>(sm, P, L.hp, ti, sm.stage[s], eb, r_s, r_v, th);
         else
-            stream_tile<TILE, THREADS, LUTR, DECR, MODE, THS, FMT, LUT, false>(sm, P, L.hp, ti, sm.stage[s], eb, r_s, r_v);
+            stream_tile<TILE, THREADS, LUTR, DECR, MODE, THS, FMT, LUT, false>(sm, P, L.hp, ti, sm.stage[s], eb, r_s, r_v, th);
 
         // every thread is done with stage s: refill it with tile it + STAGES
         if (__syncthreads_or(!ok)) {
