@@ -489,7 +489,7 @@ struct TileInfo {
     int p;
     uint32_t pmagic;  // floor(2^32 / p) + 1: e / p == umulhi(e, pmagic) for e, p < 2^16
     int ext;          // a tile of a big block: its factors were finalised beforehand
-    int pad;
+    float rp;         // 1 / p (fp32, round to nearest), computed by the issuing thread
 };
 
 template <int LUTR, int DECR>
@@ -592,7 +592,7 @@ __device__ __forceinline__ TileInfo tile_info(const Launch& L, int64_t unit, int
     const Seg& S = L.seg[seg];
     const int64_t p = S.period;
     TileInfo ti;
-    ti.pad = 0;
+    ti.rp = 0.0f;
     if (S.flags & kSegBigTiles) {
         // per_unit tiles per block, each p / per_unit consecutive elements
         const int64_t local = unit - S.unit_begin;
@@ -614,6 +614,7 @@ __device__ __forceinline__ TileInfo tile_info(const Launch& L, int64_t unit, int
     ti.e0 = S.elem_off + blk0 * p;
     ti.bo = S.block_off + blk0;
     ti.pmagic = S.pmagic;
+    ti.rp = __frcp_rn(static_cast<float>(p));
     return ti;
 }
 
@@ -756,7 +757,7 @@ __device__ __forceinline__ void stream_tile(Smem& sm, const Ptrs& P, const HP& h
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int lut_copy = lane % LUTR, dec_copy = lane % DECR;
     const int p = ti.p;
-    const float rp = __frcp_rn(static_cast<float>(p));
+    const float rp = ti.rp;
     bool live[4];
     int blk[4];
 #pragma unroll
@@ -826,10 +827,10 @@ __device__ __forceinline__ void stream_tile(Smem& sm, const Ptrs& P, const HP& h
         float s2 = warp_sum_bfly((g2[0] + g2[1]) + (g2[2] + g2[3]));
         float sx = warp_max_nonneg(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])));
         const int nw = p >> 9;  // warps per block
+        const int w0 = blk[0] * nw;  // the block's first warp (its blocks are whole warps)
         if (nw > 1) {
             if (lane == 0) sm.part[warp] = make_float2(s2, sx);
             __syncthreads();
-            const int w0 = warp - warp % nw;
             s2 = 0.0f;
             sx = 0.0f;
             for (int t = 0; t < nw; ++t) {
@@ -838,7 +839,7 @@ __device__ __forceinline__ void stream_tile(Smem& sm, const Ptrs& P, const HP& h
                 sx = fmaxf(sx, pp.y);
             }
         }
-        finish(s2, sx, r_v[0], ti.bo + blk[0], live[0] && lane == 0 && warp % nw == 0, fac[0], inv[0]);
+        finish(s2, sx, r_v[0], ti.bo + blk[0], live[0] && lane == 0 && warp == w0, fac[0], inv[0]);
 #pragma unroll
         for (int j = 1; j < 4; ++j) { fac[j] = fac[0]; inv[j] = inv[0]; }
     } else if (p == 256) {
