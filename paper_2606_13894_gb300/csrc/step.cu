@@ -516,6 +516,7 @@ struct alignas(128) StreamSmem {
     float2 part[THREADS / 32];  // per warp: (sum g^2, max |m|)
     float2 blk[TILE / 16];      // per block, irregular shapes: (step factor, 1/s')  [grad-only: (-, absmax)]
     TileInfo tile[STAGES];      // the tile each stage holds, written by the issuing thread
+    TileInfo next;              // the issuing thread's next descriptor, prepared during a tile
     unsigned long long bar[STAGES];
 };
 
@@ -833,10 +834,13 @@ __device__ __forceinline__ void stream_tile(Smem& sm, const Ptrs& P, const HP& h
             __syncthreads();
             s2 = 0.0f;
             sx = 0.0f;
-            for (int t = 0; t < nw; ++t) {
-                const float2 pp = sm.part[w0 + t];
-                s2 += pp.x;
-                sx = fmaxf(sx, pp.y);
+#pragma unroll
+            for (int t = 0; t < THREADS / 32; ++t) {
+                if (t < nw && w0 + t < THREADS / 32) {  // idle warps of a partial tile stay in range
+                    const float2 pp = sm.part[w0 + t];
+                    s2 += pp.x;
+                    sx = fmaxf(sx, pp.y);
+                }
             }
         }
         finish(s2, sx, r_v[0], ti.bo + blk[0], live[0] && lane == 0 && warp == w0, fac[0], inv[0]);
@@ -965,6 +969,13 @@ __device__ __forceinline__ void stream_loop(Smem& sm, const Launch& L, const Ptr
             if (tid == 0) atomicExch(err, 2);
             break;
         }
+        // the descriptor of the tile that refills this stage.  With two CTAs
+        // per SM (three stages) it is prepared here, off the critical path
+        // (only the issuing thread reads it back); with one CTA per SM a late
+        // warp 0 holds up the block exchange, so it is prepared after the
+        // tile's last barrier instead.
+        const int64_t un = u + static_cast<int64_t>(STAGES) * G;
+        if (STAGES >= 3 && tid == 0 && un < L.nunits) sm.next = tile_info(L, un, seg);
         // theta from global memory (an L2 hit: prefetched when the tile was
         // issued) is requested before the stage wait; from the stage, just
         // before use
@@ -1000,9 +1011,9 @@ __device__ __forceinline__ void stream_loop(Smem& sm, const Launch& L, const Ptr
             if (tid == 0) atomicExch(err, 1);
             break;
         }
-        if (tid == 0) {
-            const int64_t un = u + static_cast<int64_t>(STAGES) * G;
-            if (un < L.nunits) issue_tile<TILE, MODE, THS, FMT>(sm, s, tile_info(L, un, seg), P);
+        if (tid == 0 && un < L.nunits) {
+            if (STAGES < 3) sm.next = tile_info(L, un, seg);
+            issue_tile<TILE, MODE, THS, FMT>(sm, s, sm.next, P);
         }
         if (STAGES < 3 && MODE != kGradOnly && u + G < L.nunits)
             load_state<4>(P, sm.tile[(it + 1) % STAGES], eb, n_s, n_v);
