@@ -551,19 +551,24 @@ __global__ void __launch_bounds__(kDpWarps * 32) k_dp_levels(int B, int k, DpWs 
 }
 
 // Backtrack the splits into cell starts and levels (one thread).
+// One CTA: thread 0 follows the split positions back from (k_eff, b) -- a
+// chain of dependent loads -- and every thread then derives its levels (the
+// count-weighted mean of each run of cells, two fp64 divisions) in parallel.
 __global__ void k_dp_backtrack(int B, int k, DpWs W, float* __restrict__ codebook, int32_t* __restrict__ cell_start,
                                double* __restrict__ cost) {
-    if (threadIdx.x != 0 || blockIdx.x != 0) return;
+    if (blockIdx.x != 0) return;
+    __shared__ int start[kMaxLevels + 2];
     const Header h = *W.hdr;
     if (h.status) return;
     const int n1 = B + 1;
     const int b = h.b, ke = h.k_eff;
-    for (int j = 0; j < k; ++j) {
-        codebook[j] = 1.0f;
-        if (cell_start) cell_start[j] = -1;
-    }
-    codebook[0] = -1.0f;
     if (b <= 1) {
+        if (threadIdx.x != 0) return;
+        for (int j = 0; j < k; ++j) {
+            codebook[j] = 1.0f;
+            if (cell_start) cell_start[j] = -1;
+        }
+        codebook[0] = -1.0f;
         if (cell_start && b == 1) cell_start[0] = W.idx[1];
         if (cost) {
             double c = 0.0;
@@ -572,29 +577,38 @@ __global__ void k_dp_backtrack(int B, int k, DpWs W, float* __restrict__ codeboo
         }
         return;
     }
-    int r = b;
-    int start[kMaxLevels + 1];
-    for (int kk = ke; kk >= 1; --kk) {
-        const int l = W.A[static_cast<size_t>(kk) * n1 + r];
-        start[kk] = l;
-        r = l - 1;
+    if (threadIdx.x == 0) {
+        int r = b;
+        for (int kk = ke; kk >= 1; --kk) {
+            const int l = W.A[static_cast<size_t>(kk) * n1 + r];
+            start[kk] = l;
+            r = l - 1;
+        }
+        if (cost) *cost = W.D[static_cast<size_t>(ke) * n1 + b];
     }
-    for (int kk = 1; kk <= ke; ++kk) {
+    __syncthreads();
+    // level j = kk - 1; levels past k_eff repeat +1 (they are never the nearest)
+    for (int j = threadIdx.x; j < k; j += blockDim.x) {
+        const int kk = j + 1;
+        if (kk > ke) {
+            codebook[j] = 1.0f;
+            if (cell_start) cell_start[j] = -1;
+            continue;
+        }
         const int l = start[kk];
         const int rr = (kk == ke) ? b : start[kk + 1] - 1;
-        if (cell_start) cell_start[kk - 1] = W.idx[l];
+        if (cell_start) cell_start[j] = W.idx[l];
         if (kk == 1) {
-            codebook[0] = -1.0f;
+            codebook[j] = -1.0f;
         } else if (kk == ke) {
-            codebook[kk - 1] = 1.0f;
+            codebook[j] = 1.0f;
         } else {
             const uint64_t s0 = W.P0[rr] - W.P0[l - 1];
             const int64_t s1 = W.P1[rr] - W.P1[l - 1];
             const double mu = __ddiv_rn(__ddiv_rn(__ll2double_rn(s1), __ull2double_rn(s0)), static_cast<double>(B));
-            codebook[kk - 1] = __double2float_rn(mu);
+            codebook[j] = __double2float_rn(mu);
         }
     }
-    if (cost) *cost = W.D[static_cast<size_t>(ke) * n1 + b];
 }
 
 }  // namespace
@@ -655,7 +669,7 @@ extern "C" gefen_status_t gefen_refit_codebook(const float* x, int64_t n, const 
                                         args, 0, st) != cudaSuccess)
             return GEFEN_ECUDA;
     }
-    k_dp_backtrack<<<1, 32, 0, st>>>(bins, k, W, codebook_out, cell_start_out, cost_out);
+    k_dp_backtrack<<<1, 256, 0, st>>>(bins, k, W, codebook_out, cell_start_out, cost_out);
     if (cudaGetLastError() != cudaSuccess) return GEFEN_ECUDA;
     return GEFEN_OK;
 }
