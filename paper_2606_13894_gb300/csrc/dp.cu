@@ -550,8 +550,7 @@ __global__ void __launch_bounds__(kDpWarps * 32) k_dp_levels(int B, int k, DpWs 
     }
 }
 
-// Backtrack the splits into cell starts and levels (one thread).
-// One CTA: thread 0 follows the split positions back from (k_eff, b) -- a
+// Backtrack the splits into cell starts and levels.  One CTA: thread 0 follows the split positions back from (k_eff, b) -- a
 // chain of dependent loads -- and every thread then derives its levels (the
 // count-weighted mean of each run of cells, two fp64 divisions) in parallel.
 __global__ void k_dp_backtrack(int B, int k, DpWs W, float* __restrict__ codebook, int32_t* __restrict__ cell_start,
