@@ -394,36 +394,37 @@ def run_gpu(args, world, rank, local):
         "e2e": e2e, "gpu_launches": launches, "clocks": ck,
     }
     if rank == 0 and not args.no_microbench:
-        res["refit_microbench"] = refit_microbench(G, synth, dev)
+        res["refit_microbench"] = refit_microbench(G, synth, dev, args.micro_values, args.micro_bins)
     if rank == 0 and not args.no_cpu_baseline:
         res["cpu_baseline"] = cpu_baseline(args)
     return res
 
 
-def refit_microbench(G, synth, dev):
-    """Histogram of 1.5e9 normalised values into 65536 cells, then the exact DP
-    to 256 levels; CUDA-event times of each part (after one untimed run)."""
-    x = synth.refit_values(MICRO_N, SEED + 7, device=dev)
-    hist = torch.zeros(MICRO_BINS, dtype=torch.int64, device=dev)
+def refit_microbench(G, synth, dev, n=MICRO_N, bins=MICRO_BINS):
+    """Histogram of n normalised values (default 1.5e9) into `bins` cells
+    (default 65536), then the exact DP to 256 levels; CUDA-event times of each
+    part (after one untimed run)."""
+    x = synth.refit_values(n, SEED + 7, device=dev)
+    hist = torch.zeros(bins, dtype=torch.int64, device=dev)
     cb = torch.empty(K, dtype=torch.float32, device=dev)
-    ws = G.workspace(G.gefen_refit_workspace_size(MICRO_BINS, K), dev)
-    G.gefen_refit_codebook(bins=MICRO_BINS, k=K, codebook_out=cb, x=x, hist_out=hist, workspace_buf=ws)
+    ws = G.workspace(G.gefen_refit_workspace_size(bins, K), dev)
+    G.gefen_refit_codebook(bins=bins, k=K, codebook_out=cb, x=x, hist_out=hist, workspace_buf=ws)
     torch.cuda.synchronize()
     e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
     e[0].record()
-    G.gefen_refit_codebook(bins=MICRO_BINS, k=K, codebook_out=cb, x=x, hist_out=hist, workspace_buf=ws)
+    G.gefen_refit_codebook(bins=bins, k=K, codebook_out=cb, x=x, hist_out=hist, workspace_buf=ws)
     e[1].record()
-    G.gefen_refit_codebook(bins=MICRO_BINS, k=K, codebook_out=cb, hist_in=hist, workspace_buf=ws)
+    G.gefen_refit_codebook(bins=bins, k=K, codebook_out=cb, hist_in=hist, workspace_buf=ws)
     e[2].record()
     torch.cuda.synchronize()
     ke = G.gefen_refit_status(ws)
     hist_dp_ms, dp_ms = e[0].elapsed_time(e[1]), e[1].elapsed_time(e[2])
     del x
     torch.cuda.empty_cache()
-    return {"values": MICRO_N, "bins": MICRO_BINS, "levels": K, "k_eff": ke,
+    return {"values": n, "bins": bins, "levels": K, "k_eff": ke,
             "nonempty_cells": int((hist > 0).sum().item()),
             "hist_ms": hist_dp_ms - dp_ms, "dp_ms": dp_ms, "total_ms": hist_dp_ms,
-            "hist_gbs": 4 * MICRO_N / ((hist_dp_ms - dp_ms) * 1e-3) / 1e9}
+            "hist_gbs": 4 * n / ((hist_dp_ms - dp_ms) * 1e-3) / 1e9}
 
 
 def run_e2e(G, table, theta, codes, v, sc, cb, ws, gpool, nparams, stream, args, state, one_step_ctx):
@@ -559,9 +560,21 @@ def main():
     ap.add_argument("--ref-params", type=float, default=20e6, help="oracle params per reference step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-microbench", action="store_true", help="skip the 65536-cell refit measurement")
+    ap.add_argument("--microbench-only", action="store_true",
+                    help="run only the refit micro-benchmark and print its figures (one GPU)")
+    ap.add_argument("--micro-values", type=int, default=MICRO_N, help="refit micro-benchmark values (multiple of 4096)")
+    ap.add_argument("--micro-bins", type=int, default=MICRO_BINS, help="refit micro-benchmark histogram cells")
     ap.add_argument("--workload", default=WORKLOAD,
                     help="llama-1.5b (default), gpt2-125m, tiny, or flat:N:P (one tensor, blocks of P)")
     args = ap.parse_args()
+    if args.microbench_only:
+        from paper_2606_13894_gb300 import gefen as G
+        from paper_2606_13894_gb300 import synth
+        G.load()
+        dev = torch.device("cuda", 0)
+        print(json.dumps({"refit_microbench": refit_microbench(G, synth, dev, args.micro_values, args.micro_bins)}),
+              flush=True)
+        return
     world, rank, local = dist_env()
     if args.impl == "reference":
         res = run_reference(args, world, rank)

@@ -1395,7 +1395,7 @@ using S8KCfg = StreamCfg<8192, 512, 2, 8, 32, true, 1>;
 // Steps that also histogram x (refit steps) count up to kFusedBins cells in
 // shared memory; the tables give up copies to make room.
 constexpr int kFusedBins = 4096;
-using S4KHistCfg = StreamCfg<4096, 256, 3, 2, 4, false, 2>;
+using S4KHistCfg = StreamCfg<4096, 256, 3, 4, 8, false, 2>;
 using S8KHistCfg = StreamCfg<8192, 512, 2, 2, 4, true, 1>;
 constexpr int kS4KTile = S4KCfg::TILE, kS8KTile = S8KCfg::TILE;
 
