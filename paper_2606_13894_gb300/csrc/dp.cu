@@ -389,10 +389,10 @@ __device__ __forceinline__ void settle(const RowCtx& c, Search& S) {
     S.pl = 0;
 }
 
-// One round over up to 32 candidates a, a+st, ..., one per lane, up to e.
-__device__ __forceinline__ void eval_candidates(const RowCtx& c, int a, int e, int lane, Search& S, int st = 1) {
-    const int l = a + lane * st;
-    const bool in = l <= e;
+// One round over up to 32 candidates, one per lane (l = 0: none; every
+// candidate is >= 2).
+__device__ __forceinline__ void eval_lanes(const RowCtx& c, int l, Search& S) {
+    const bool in = l != 0;
     ff v{INFINITY, 0.0f};
     if (in) v = ff_add(ld_ff(c.Ep, l), run_cost_ff(c, l));
     const ff vm = warp_min_ff(v);
@@ -402,6 +402,11 @@ __device__ __forceinline__ void eval_candidates(const RowCtx& c, int a, int e, i
         S.pl = l;
         S.pv = v;
     }
+}
+// One round over the candidates a, a+st, ..., up to e (at most 32).
+__device__ __forceinline__ void eval_candidates(const RowCtx& c, int a, int e, int lane, Search& S, int st = 1) {
+    const int l = a + lane * st;
+    eval_lanes(c, l <= e ? l : 0, S);
 }
 
 __device__ Best search_row(const RowCtx& c, int kk, int hint, int lane, int2* stack) {
@@ -431,13 +436,25 @@ __device__ Best search_row(const RowCtx& c, int kk, int hint, int lane, int2* st
     sp = (w1 < r ? 1 : 0) + (w0 > kk ? 1 : 0);
     __syncwarp();
     while (sp > 0) {
+        if (stack[sp - 1].y - stack[sp - 1].x < 32) {
+            // runs of at most 32 candidates from the top of the stack, packed
+            // into one round as long as they fit
+            int n = 0, l = 0;
+            while (sp > 0) {
+                const int2 q = stack[sp - 1];
+                const int w = q.y - q.x + 1;
+                if (n + w > 32) break;
+                if (lane >= n && lane < n + w) l = q.x + (lane - n);
+                n += w;
+                --sp;
+            }
+            __syncwarp();
+            eval_lanes(c, l, S);
+            continue;
+        }
         const int2 run = stack[--sp];
         __syncwarp();
         const int a = run.x, e = run.y, width = e - a + 1;
-        if (width <= 32) {
-            eval_candidates(c, a, e, lane, S);
-            continue;
-        }
         // 32 sub-runs; lane i bounds [ca, ce] by D[ca-1] + cost(ce..r)
         const int cw = (width + 31) >> 5;
         const int ca = a + lane * cw, ce = min(e, ca + cw - 1);
