@@ -8,7 +8,8 @@
 //   last      (double)(s2 - 2B s1 + B^2 s0)      (centre +1)
 // D[r][k'] = min_{k' <= l <= r} D[l-1][k'-1] + cost(l..r), ties to the smallest l.
 //
-// One launch per level, one warp per end position r.  fp64 is slow on this
+// Levels 2..k in one cooperative launch with a grid barrier between levels,
+// one warp per end position r at a time.  fp64 is slow on this
 // part, so candidates are screened in float-float arithmetic (a pair of fp32
 // values, about 2^-43 relative error): D[.][k'-1] is kept as a (hi, lo) pair
 // and each cost comes from its exact 128-bit integer numerator.  Whole runs of
@@ -18,9 +19,11 @@
 // cost less).  So for l in [a, e]:  value(l) >= D[a-1][k'-1] + cost(e..r).
 // A 32-wide window around a hint (the previous level's split at r, moved by
 // its share of the last cell; on level 2, the best of 32 evenly spaced
-// candidates) gives the best screened value u, one candidate per lane; the rest of [k', r] is searched by 32-way subdivision (one run
-// bound per lane), dropping every run whose bound exceeds u by more than 2^-34
-// relative.  Survivors (near-ties only) get the
+// candidates) gives the best screened value u, one candidate per lane; the
+// rest of [k', r] is searched by 32-way subdivision (one run bound per lane),
+// dropping every run whose bound exceeds u by more than 2^-34 relative, and
+// the narrow runs left are screened 32 candidates to a round.  Survivors
+// (near-ties only) get the
 // canonical fp64 value once the final bound is known; their minimum, ties to
 // the smallest l, equals the full scan bit for bit.
 #include <algorithm>
