@@ -24,7 +24,9 @@ def _refit_from_hist(h, k):
     return cbo.cpu().numpy(), cs.cpu().numpy(), float(cost.cpu()[0]), ke, ws
 
 
-@pytest.mark.parametrize("bins", [16, 4096, 65536, 1000])
+# 16385 and 65535: the two CTAs of a cell-splitting pair own halves that
+# differ by one cell
+@pytest.mark.parametrize("bins", [16, 4096, 65536, 1000, 16385, 65535])
 @pytest.mark.parametrize("n", [0, 1, 7, 100_003, 3_000_001])
 def test_histogram_bit_exact(bins, n):
     rng = np.random.default_rng(n + bins)
@@ -37,6 +39,33 @@ def test_histogram_bit_exact(bins, n):
     G.gefen_refit_codebook(bins=bins, k=4, codebook_out=cbo, x=xd, hist_out=ho)
     ref = oracle.histogram(x, bins)
     np.testing.assert_array_equal(ho.cpu().numpy().astype(np.uint64), ref)
+
+
+@pytest.mark.parametrize("bins", [4096, 65536])
+@pytest.mark.parametrize("offset", [0, 4])
+def test_histogram_one_cell(bins, offset):
+    # every value in one cell (x = 0 and its neighbours within the cell), a
+    # start past the array's first element, counts far above 2^16 per CTA
+    n = 5_000_003
+    x = np.zeros(n + offset, np.float32)
+    x[offset + 1::7] = np.float32(0.25 / bins)
+    x[offset + 2::11] = -0.0
+    xd = torch.from_numpy(x).cuda()[offset:]
+    ho = torch.zeros(bins, dtype=torch.int64, device="cuda")
+    cbo = torch.empty(4, dtype=torch.float32, device="cuda")
+    G.gefen_refit_codebook(bins=bins, k=4, codebook_out=cbo, x=xd, hist_out=ho)
+    ref = oracle.histogram(x[offset:], bins)
+    assert ref.max() == n
+    np.testing.assert_array_equal(ho.cpu().numpy().astype(np.uint64), ref)
+
+
+def test_histogram_input_must_be_16_byte_aligned():
+    # rejected on the host before any launch
+    xd = torch.zeros(1027, dtype=torch.float32, device="cuda")[3:]
+    ho = torch.zeros(4096, dtype=torch.int64, device="cuda")
+    cbo = torch.empty(4, dtype=torch.float32, device="cuda")
+    with pytest.raises(G.GefenError):
+        G.gefen_refit_codebook(bins=4096, k=4, codebook_out=cbo, x=xd, hist_out=ho)
 
 
 def _t_hist(B, n, seed):
