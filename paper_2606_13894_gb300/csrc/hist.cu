@@ -174,14 +174,19 @@ cudaError_t launch_histogram(const float* x, const HistRange* ranges, int nrange
             if (e != cudaSuccess) return e;
             // all clusters co-resident (units are dealt out statically): the
             // number of SM pairs the hardware can place, not sms / 2
-            int fit = 0;
-            cudaLaunchConfig_t cfg = {};
-            cfg.gridDim = dim3(2 * static_cast<unsigned>(std::max(1, sms / 2)));
-            cfg.blockDim = dim3(kHistThreads);
-            cfg.dynamicSmemBytes = smem;
-            if (cudaOccupancyMaxActiveClusters(&fit, k_hist2, &cfg) != cudaSuccess || fit < 1) {
-                (void)cudaGetLastError();
-                fit = std::max(1, sms / 2);
+            // (a property of the kernel and its shared memory: asked once per size)
+            static thread_local size_t fit_smem = 0;
+            static thread_local int fit = 0;
+            if (fit_smem != smem) {
+                cudaLaunchConfig_t cfg = {};
+                cfg.gridDim = dim3(2 * static_cast<unsigned>(std::max(1, sms / 2)));
+                cfg.blockDim = dim3(kHistThreads);
+                cfg.dynamicSmemBytes = smem;
+                if (cudaOccupancyMaxActiveClusters(&fit, k_hist2, &cfg) != cudaSuccess || fit < 1) {
+                    (void)cudaGetLastError();
+                    fit = std::max(1, sms / 2);
+                }
+                fit_smem = smem;
             }
             const int64_t clusters = std::min<int64_t>(units, fit);
             k_hist2<<<dim3(static_cast<unsigned>(2 * clusters)), kHistThreads, smem, stream>>>(x, L, hist);

@@ -71,21 +71,39 @@ struct MuonArgs {
     void* u;  // update buffer (fp32 or bf16)
 };
 
-__device__ __forceinline__ float muon_m(const MuonArgs& A, const float* s_dec, int64_t e) {
+// Block of element e (a 32-bit division whenever n < 2^32, the usual case).
+__device__ __forceinline__ int64_t muon_block(const MuonArgs& A, int64_t e) {
+    if (A.n < (int64_t(1) << 32))
+        return static_cast<uint32_t>(e) / static_cast<uint32_t>(A.period);
+    return e / A.period;
+}
+
+__device__ __forceinline__ float muon_m(const MuonArgs& A, const float* s_dec, int64_t e, int64_t bi) {
     const float g = bf16_bits_to_f32(A.grads[e]);
-    return fmaf(A.omm, g, A.mu * A.scale[e / A.period] * s_dec[A.codes[e]]);
+    return fmaf(A.omm, g, A.mu * A.scale[bi] * s_dec[A.codes[e]]);
 }
 
 // s'_b = max |m| over each block (atomic max of non-negative float bits:
-// exact and order-independent).
+// exact and order-independent).  A warp whose 32 elements lie in one block
+// takes their maximum first and sends one atomic.
 __global__ void __launch_bounds__(kMuThreads) k_muon_absmax(MuonArgs A) {
     __shared__ float s_dec[kMaxLevels];
     if (threadIdx.x < kMaxLevels) s_dec[threadIdx.x] = threadIdx.x < A.k ? A.cb_dec[threadIdx.x] : 0.0f;
     __syncthreads();
     for (int64_t e = blockIdx.x * static_cast<int64_t>(kMuThreads) + threadIdx.x; e < A.n;
          e += static_cast<int64_t>(gridDim.x) * kMuThreads) {
-        const float am = fabsf(muon_m(A, s_dec, e));
-        atomicMax(reinterpret_cast<unsigned int*>(A.snew) + e / A.period, __float_as_uint(am));
+        const int64_t bi = muon_block(A, e);
+        const unsigned am = __float_as_uint(fabsf(muon_m(A, s_dec, e, bi)));
+        unsigned* dst = reinterpret_cast<unsigned int*>(A.snew) + bi;
+        const unsigned live = __activemask();
+        const int first = __ffs(live) - 1;
+        const long long b0 = __shfl_sync(live, static_cast<long long>(bi), first);
+        if (__all_sync(live, bi == b0)) {
+            const unsigned wm = __reduce_max_sync(live, am);
+            if ((threadIdx.x & 31) == first) atomicMax(dst, wm);
+        } else {
+            atomicMax(dst, am);
+        }
     }
 }
 
@@ -104,9 +122,10 @@ __global__ void __launch_bounds__(kMuThreads) k_muon_encode(MuonArgs A) {
     double acc = 0.0;
     for (int64_t e = blockIdx.x * static_cast<int64_t>(kMuThreads) + t; e < A.n;
          e += static_cast<int64_t>(gridDim.x) * kMuThreads) {
+        const int64_t bi = muon_block(A, e);
         const float g = bf16_bits_to_f32(A.grads[e]);
-        const float m = fmaf(A.omm, g, A.mu * A.scale[e / A.period] * s_dec[A.codes[e]]);
-        const float sn = A.snew[e / A.period];
+        const float m = fmaf(A.omm, g, A.mu * A.scale[bi] * s_dec[A.codes[e]]);
+        const float sn = A.snew[bi];
         A.codes[e] = static_cast<uint8_t>(sn > 0.0f ? level_search(s_mid, __fdiv_rn(m, sn)) : zero_code);
         const float u = A.nesterov ? fmaf(A.mu, m - g, g) : m;
         if (BF16) {
@@ -130,15 +149,22 @@ __global__ void __launch_bounds__(kMuThreads) k_muon_encode(MuonArgs A) {
     }
 }
 
-// Normalise U (one fixed-order sum of the partials) and commit the new scales.
+// Normalise U and commit the new scales.  Every CTA sums the partials in the
+// same fixed order (thread t: partials t, t + 256, ...; then a fixed tree),
+// so all use the same norm.
 template <bool BF16>
 __global__ void __launch_bounds__(kMuThreads) k_muon_normalise(MuonArgs A, int nparts, double eps) {
+    __shared__ double s_sum[kMuThreads];
     __shared__ float s_inv;
-    if (threadIdx.x == 0) {
-        double s = 0.0;
-        for (int i = 0; i < nparts; ++i) s += A.part[i];
-        s_inv = static_cast<float>(1.0 / fmax(sqrt(s), eps));
+    double ps = 0.0;
+    for (int i = threadIdx.x; i < nparts; i += kMuThreads) ps += A.part[i];
+    s_sum[threadIdx.x] = ps;
+    __syncthreads();
+    for (int w = kMuThreads / 2; w > 0; w >>= 1) {
+        if (threadIdx.x < w) s_sum[threadIdx.x] += s_sum[threadIdx.x + w];
+        __syncthreads();
     }
+    if (threadIdx.x == 0) s_inv = static_cast<float>(1.0 / fmax(sqrt(s_sum[0]), eps));
     __syncthreads();
     const float inv = s_inv;
     const int64_t nb = A.n / A.period;
