@@ -2,21 +2,17 @@
 // entries of Z into histogram counts").
 //
 // HBM-bound: 4 bytes read per value.  Counts are privatised in shared memory
-// (u32) and flushed to the u64 result once per CTA.  Up to 16384 cells fit in
-// one CTA; for up to 65536 cells a cluster of two CTAs splits the cells, each
-// CTA owning half in its shared memory.  Both CTAs of the pair read every value
-// of their unit (the second read is an L2 hit: the pair runs together) and each
-// counts only the values of its own cells, so no count crosses between CTAs.
-// NaN values are skipped.
-#include <cooperative_groups.h>
-
+// and flushed to the u64 result once per CTA.  Up to 16384 cells: u32
+// counters.  Up to 65536 cells: two 16-bit counters per u32 word (128 KB for
+// 65536 cells, one CTA per SM), kept below 2^16 by construction: after every
+// kPackedUnits units (at most 49152 values) the CTA moves each counter that
+// has reached 2^14 to the u64 result, so between checks none can pass
+// 2^14 - 1 + 49152 = 65535.  NaN values are skipped.
 #include <algorithm>
 #include <vector>
 
 #include "common.cuh"
 #include "internal.h"
-
-namespace cg = cooperative_groups;
 
 namespace gefen {
 
@@ -26,6 +22,9 @@ constexpr int kHistThreads = 1024;
 constexpr int kHistMaxRanges = 512;
 constexpr int64_t kHistUnit = 16384;  // values per work unit
 constexpr int kHistLoads = 4;         // float4 loads in flight per thread
+constexpr int kPacked = 16;           // hist_body mode: two 16-bit counters per word
+constexpr int kPackedUnits = 3;       // units between checks of the 16-bit counters
+constexpr unsigned kSpillAt = 1u << 14;
 
 struct HistLaunch {
     int32_t nranges;
@@ -46,27 +45,43 @@ __device__ __forceinline__ int find_range(const HistLaunch& L, int64_t unit) {
 }
 
 template <int CL>
-__device__ __forceinline__ void count_one(float x, float halfB, int B, int per, unsigned* local, unsigned rank) {
+__device__ __forceinline__ void count_one(float x, float halfB, int B, unsigned* local) {
     if (isnan(x)) return;
     const int c = hist_cell(x, halfB, B);
-    if (CL == 1) {
+    if (CL == kPacked)
+        atomicAdd(local + (c >> 1), 1u << ((c & 1) << 4));  // cell c: half c & 1 of word c / 2
+    else
         atomicAdd(local + c, 1u);
-    } else {
-        const int li = c - static_cast<int>(rank) * per;  // this CTA's cells: [rank per, (rank+1) per)
-        if (static_cast<unsigned>(li) < static_cast<unsigned>(per)) atomicAdd(local + li, 1u);
+}
+
+// Moves every 16-bit counter that has reached kSpillAt to the u64 result
+// (between two CTA barriers: no count is in flight).
+__device__ __forceinline__ void spill_packed(unsigned* words, int B, uint64_t* __restrict__ hist) {
+    const int nw = (B + 1) >> 1;
+    for (int i = threadIdx.x; i < nw; i += blockDim.x) {
+        const unsigned w = words[i];
+        const unsigned lo = w & 0xFFFFu, hi = w >> 16;
+        if (lo < kSpillAt && hi < kSpillAt) continue;
+        unsigned keep = w;
+        if (lo >= kSpillAt) {
+            atomicAdd(reinterpret_cast<unsigned long long*>(hist + 2 * i), static_cast<unsigned long long>(lo));
+            keep &= 0xFFFF0000u;
+        }
+        if (hi >= kSpillAt) {
+            atomicAdd(reinterpret_cast<unsigned long long*>(hist + 2 * i + 1), static_cast<unsigned long long>(hi));
+            keep &= 0x0000FFFFu;
+        }
+        words[i] = keep;
     }
 }
 
 template <int CL>
 __device__ __forceinline__ void hist_body(const float* __restrict__ x, const HistLaunch& L,
-                                          uint64_t* __restrict__ hist, unsigned* s_hist, unsigned rank) {
+                                          uint64_t* __restrict__ hist, unsigned* s_hist) {
     const int B = L.bins;
-    const int per = (B + CL - 1) / CL;  // cells owned by each CTA of the cluster
     const float halfB = 0.5f * static_cast<float>(B);
-    const int64_t nclusters = gridDim.x / CL;
-    const int64_t cid = blockIdx.x / CL;
-    // every CTA of a cluster reads the whole unit
-    for (int64_t u = cid; u < L.nunits; u += nclusters) {
+    int since = 0;  // units since the last check of the 16-bit counters (uniform)
+    for (int64_t u = blockIdx.x; u < L.nunits; u += gridDim.x) {
         const int r = find_range(L, u);
         const int64_t s0 = L.off[r] + (u - L.unit_begin[r]) * kHistUnit;
         const int64_t s1 = min(s0 + kHistUnit, L.off[r] + L.cnt[r]);
@@ -75,7 +90,7 @@ __device__ __forceinline__ void hist_body(const float* __restrict__ x, const His
         int64_t h = (s0 + 3) & ~int64_t(3);
         if (h > s1) h = s1;
         for (int64_t e = s0 + threadIdx.x; e < h; e += blockDim.x)
-            count_one<CL>(__ldcg(x + e), halfB, B, per, s_hist, rank);
+            count_one<CL>(__ldcg(x + e), halfB, B, s_hist);
         const int64_t nv = (s1 - h) >> 2;
         const float4* xv = reinterpret_cast<const float4*>(x + h);
         // kHistLoads float4 loads in flight per thread before any count (a
@@ -89,14 +104,20 @@ __device__ __forceinline__ void hist_body(const float* __restrict__ x, const His
             }
 #pragma unroll
             for (int u = 0; u < kHistLoads; ++u) {
-                count_one<CL>(q[u].x, halfB, B, per, s_hist, rank);
-                count_one<CL>(q[u].y, halfB, B, per, s_hist, rank);
-                count_one<CL>(q[u].z, halfB, B, per, s_hist, rank);
-                count_one<CL>(q[u].w, halfB, B, per, s_hist, rank);
+                count_one<CL>(q[u].x, halfB, B, s_hist);
+                count_one<CL>(q[u].y, halfB, B, s_hist);
+                count_one<CL>(q[u].z, halfB, B, s_hist);
+                count_one<CL>(q[u].w, halfB, B, s_hist);
             }
         }
         for (int64_t e = h + nv * 4 + threadIdx.x; e < s1; e += blockDim.x)
-            count_one<CL>(__ldcg(x + e), halfB, B, per, s_hist, rank);
+            count_one<CL>(__ldcg(x + e), halfB, B, s_hist);
+        if (CL == kPacked && ++since == kPackedUnits) {
+            since = 0;
+            __syncthreads();
+            spill_packed(s_hist, B, hist);
+            __syncthreads();
+        }
     }
 }
 
@@ -106,7 +127,7 @@ __global__ void __launch_bounds__(kHistThreads) k_hist1(const float* __restrict_
     const int B = L.bins;
     for (int i = threadIdx.x; i < B; i += blockDim.x) s_hist[i] = 0u;
     __syncthreads();
-    hist_body<1>(x, L, hist, s_hist, 0u);
+    hist_body<1>(x, L, hist, s_hist);
     __syncthreads();
     for (int i = threadIdx.x; i < B; i += blockDim.x) {
         const unsigned c = s_hist[i];
@@ -114,21 +135,22 @@ __global__ void __launch_bounds__(kHistThreads) k_hist1(const float* __restrict_
     }
 }
 
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kHistThreads)
-    k_hist2(const float* __restrict__ x, const __grid_constant__ HistLaunch L, uint64_t* __restrict__ hist) {
-    extern __shared__ unsigned s_hist[];
-    cg::cluster_group cluster = cg::this_cluster();
-    const unsigned rank = cluster.block_rank();
+__global__ void __launch_bounds__(kHistThreads) k_hist16(const float* __restrict__ x,
+                                                        const __grid_constant__ HistLaunch L,
+                                                        uint64_t* __restrict__ hist) {
+    extern __shared__ unsigned s_words[];  // cell c: half c & 1 of word c / 2
     const int B = L.bins;
-    const int per = (B + 1) / 2;
-    for (int i = threadIdx.x; i < per; i += blockDim.x) s_hist[i] = 0u;
+    const int nw = (B + 1) >> 1;
+    for (int i = threadIdx.x; i < nw; i += blockDim.x) s_words[i] = 0u;
     __syncthreads();
-    hist_body<2>(x, L, hist, s_hist, rank);
+    hist_body<kPacked>(x, L, hist, s_words);
     __syncthreads();
-    const int base = static_cast<int>(rank) * per;
-    for (int i = threadIdx.x; i < per && base + i < B; i += blockDim.x) {
-        const unsigned c = s_hist[i];
-        if (c) atomicAdd(reinterpret_cast<unsigned long long*>(hist + base + i), static_cast<unsigned long long>(c));
+    for (int i = threadIdx.x; i < nw; i += blockDim.x) {
+        const unsigned w = s_words[i];
+        const unsigned lo = w & 0xFFFFu, hi = w >> 16;
+        if (lo) atomicAdd(reinterpret_cast<unsigned long long*>(hist + 2 * i), static_cast<unsigned long long>(lo));
+        if (hi && 2 * i + 1 < B)
+            atomicAdd(reinterpret_cast<unsigned long long*>(hist + 2 * i + 1), static_cast<unsigned long long>(hi));
     }
 }
 
@@ -137,7 +159,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kHistThreads)
 cudaError_t launch_histogram(const float* x, const HistRange* ranges, int nranges, int bins, uint64_t* hist,
                              cudaStream_t stream) {
     // One launch sees at most 2^36 values, so a CTA's u32 counters (it handles
-    // a 1/(number of clusters) share) stay far below 2^32.
+    // a 1/(number of CTAs) share) stay far below 2^32.
     constexpr int64_t kMaxPerLaunch = int64_t(1) << 36;
     static thread_local HistLaunch L;
     const int sms = device_sm_count();
@@ -170,26 +192,21 @@ cudaError_t launch_histogram(const float* x, const HistRange* ranges, int nrange
             k_hist1<<<dim3(static_cast<unsigned>(grid)), kHistThreads, smem, stream>>>(x, L, hist);
         } else {
             const size_t smem = static_cast<size_t>((bins + 1) / 2) * sizeof(unsigned);
-            e = cudaFuncSetAttribute(k_hist2, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+            e = cudaFuncSetAttribute(k_hist16, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
             if (e != cudaSuccess) return e;
-            // all clusters co-resident (units are dealt out statically): the
-            // number of SM pairs the hardware can place, not sms / 2
-            // (a property of the kernel and its shared memory: asked once per size)
+            // resident CTAs per SM for this size (asked once per size)
             static thread_local size_t fit_smem = 0;
-            static thread_local int fit = 0;
+            static thread_local int per_sm = 1;
             if (fit_smem != smem) {
-                cudaLaunchConfig_t cfg = {};
-                cfg.gridDim = dim3(2 * static_cast<unsigned>(std::max(1, sms / 2)));
-                cfg.blockDim = dim3(kHistThreads);
-                cfg.dynamicSmemBytes = smem;
-                if (cudaOccupancyMaxActiveClusters(&fit, k_hist2, &cfg) != cudaSuccess || fit < 1) {
+                if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_hist16, kHistThreads, smem) !=
+                        cudaSuccess || per_sm < 1) {
                     (void)cudaGetLastError();
-                    fit = std::max(1, sms / 2);
+                    per_sm = 1;
                 }
                 fit_smem = smem;
             }
-            const int64_t clusters = std::min<int64_t>(units, fit);
-            k_hist2<<<dim3(static_cast<unsigned>(2 * clusters)), kHistThreads, smem, stream>>>(x, L, hist);
+            const int64_t grid = std::min<int64_t>(units, static_cast<int64_t>(per_sm) * sms);
+            k_hist16<<<dim3(static_cast<unsigned>(grid)), kHistThreads, smem, stream>>>(x, L, hist);
         }
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
