@@ -32,12 +32,16 @@ def test_bin_edges_by_hand(B):
                 assert oracle.bin_index(float(below), B) == i - 1
 
 
-def test_histogram_matches_numpy_away_from_edges():
-    rng = np.random.default_rng(0)
-    B = 4096
+@pytest.mark.parametrize("B", [4096, 1000, 16385, 65535])
+def test_histogram_matches_numpy_away_from_edges(B):
+    # odd B: the cell edges are not fp32 values, so only values clear of them
+    # have a cell that does not depend on rounding
+    rng = np.random.default_rng(B)
     x = np.clip(rng.standard_t(4, 300_000) / 12, -1, 1).astype(np.float32)
     t = (x.astype(np.float64) + 1) * B / 2
-    keep = np.abs(t - np.round(t)) > 1e-3  # clear of cell edges
+    # clear of cell edges by more than the two fp32 roundings of the cell
+    # definition can move t (each at most 2^-24 relative: together < B 2^-23)
+    keep = np.abs(t - np.round(t)) > max(1e-3, B * 2.0 ** -21)
     x = x[keep]
     h = oracle.histogram(x, B)
     ref, _ = np.histogram(x.astype(np.float64), bins=B, range=(-1.0, 1.0))
