@@ -11,7 +11,8 @@
  *  - The caller owns every buffer.  The library never allocates device memory:
  *    scratch comes from a caller-provided workspace whose size the matching
  *    *_workspace_size() call returns (0 means none is needed; a NULL workspace
- *    is then allowed).  Calls keep no state between invocations.
+ *    is then allowed).  Calls keep no state between invocations, except the
+ *    static refit's own array and the refit's test hook (both below).
  *  - All work is enqueued on `stream` (a cudaStream_t; NULL is the legacy
  *    default stream) and returns without waiting, unless a call's description
  *    says it synchronises.
@@ -40,7 +41,7 @@ typedef enum {
     GEFEN_EINVAL = 1,       /* bad argument (host-side check, nothing enqueued) */
     GEFEN_ECUDA = 2,        /* a CUDA runtime call or kernel launch failed */
     GEFEN_ENOMEM = 3,       /* workspace smaller than the size query requires */
-    GEFEN_ETIMEOUT = 4,     /* reserved: a bounded device wait expired */
+    GEFEN_ETIMEOUT = 4,     /* a bounded device wait gave up (the call's outputs are not valid) */
     GEFEN_EUNSUPPORTED = 5, /* not an sm_103 device, or a size past a stated limit */
     GEFEN_EDEVICE = 6       /* the device-side check of a call's data failed */
 } gefen_status_t;
@@ -175,9 +176,11 @@ gefen_status_t gefen_step_status(void* workspace, gefen_stream_t stream);
  * cost_out       f64[1] device, nullable: the optimum D[b][k_eff].
  * Requirements: 1 <= bins <= GEFEN_MAX_BINS, 2 <= k <= GEFEN_MAX_LEVELS,
  * n >= 0, x 16-byte aligned, total count N < 2^62 with N*(bins-1)^2 < 2^64
- * (checked on the device: on
- * failure the outputs are left untouched and gefen_refit_status() reports
- * GEFEN_EDEVICE).  workspace: gefen_refit_workspace_size() bytes.
+ * (checked on the device: on failure the outputs are left untouched and
+ * gefen_refit_status() reports GEFEN_EDEVICE).  The DP's levels are separated
+ * by grid-wide barriers whose waits are bounded (about a second); if one gives
+ * up, the outputs are left untouched and gefen_refit_status() reports
+ * GEFEN_ETIMEOUT.  workspace: gefen_refit_workspace_size() bytes.
  * ------------------------------------------------------------------------- */
 size_t gefen_refit_workspace_size(int32_t bins, int32_t k);
 gefen_status_t gefen_refit_codebook(const float* x, int64_t n, const uint64_t* hist_in,
@@ -189,8 +192,8 @@ gefen_status_t gefen_refit_codebook(const float* x, int64_t n, const uint64_t* h
 /* Device-side status of the last gefen_refit_codebook() that used this
  * workspace; synchronises `stream`.  k_eff_out (host, nullable) receives the
  * number of levels the DP used.  GEFEN_EDEVICE: the moment bound above was
- * exceeded; GEFEN_ETIMEOUT: a bounded wait between DP levels gave up (the
- * outputs are then undefined). */
+ * exceeded; GEFEN_ETIMEOUT: a bounded wait between DP levels gave up.  Either
+ * way the codebook, cell starts and cost were left untouched. */
 gefen_status_t gefen_refit_status(const void* workspace, int32_t* k_eff_out,
                                   gefen_stream_t stream);
 
@@ -202,6 +205,19 @@ gefen_status_t gefen_refit_tables(const void* workspace, int32_t bins, int32_t k
                                   double* dtable_out, int32_t* argl_out,
                                   gefen_stream_t stream);
 
+/* Test hook of gefen_refit_codebook (the paper has no counterpart): a
+ * process-wide setting read by every later refit launch.
+ * anchor_stride: -1 chooses automatically (the default), 0 searches every end
+ * position over its whole range, s >= 1 puts an anchor every s positions
+ * (results are identical in every case).  barrier_extra: 0 normally; any other
+ * value makes every level barrier wait for arrivals that never come, so the
+ * refit gives up after barrier_spin_cycles (0: the default of about 2^31
+ * cycles) and gefen_refit_status() reports GEFEN_ETIMEOUT.  Call it again
+ * with (-1, 0, 0) to restore the defaults.  Not for concurrent use with
+ * refits on other threads. */
+gefen_status_t gefen_refit_debug(int32_t anchor_stride, uint32_t barrier_extra,
+                                 int64_t barrier_spin_cycles);
+
 /* -------------------------------------------------------------------------
  * gefen_refit_codebook_static -- gefen_refit_codebook without a workspace.
  * The paper has no counterpart: this entry point exists for callers that
@@ -212,22 +228,31 @@ gefen_status_t gefen_refit_tables(const void* workspace, int32_t bins, int32_t k
  *
  * Same inputs, outputs and results as gefen_refit_codebook(); the scratch is
  * one device array inside the library, sized for bins <= 4096 and k <= 256
- * (about 21.2 MB, held on every device that loads the library until the
- * process exits).  Larger requests return GEFEN_EUNSUPPORTED.  It allocates
- * nothing: no cudaMalloc, cudaFree or allocating library call.
+ * (about 21.5 MB).  Larger requests return GEFEN_EUNSUPPORTED.  The call
+ * allocates nothing: no cudaMalloc, cudaFree or allocating library call.
  *
- * The first call on a device looks up the array's device address for that
- * device (once), so make it before any stream capture on that device.  All
- * calls share the one array and it keeps the last call's contents (the refit
- * clears what it needs); calls whose work overlaps on the GPU -- different
- * streams, or different host threads -- race on it and must be ordered by the
- * caller.  The device-side overflow check of the moments is not reported by
- * this entry point; gefen_refit_codebook() with gefen_refit_status() reports it.
+ * The array exists on a device once the library's refit module is loaded
+ * there, which CUDA's lazy loading delays to the first use, and it stays
+ * until the process exits.  So call gefen_refit_static_init() once per device
+ * (with that device current) before a caching allocator or runtime reserves
+ * the device's memory, and before any stream capture: it loads the module,
+ * looks up the array's device address and loads the refit's kernels.
+ * Otherwise the first gefen_refit_codebook_static() on a device does the same.
+ * All calls share the one array and it keeps the last call's contents (the
+ * refit clears what it needs); calls whose work overlaps on the GPU --
+ * different streams, or different host threads -- race on it and must be
+ * ordered by the caller.
+ * gefen_refit_static_status() reads the device-side status of the last static
+ * refit (synchronises `stream`): GEFEN_EDEVICE if the moment bound was
+ * exceeded, GEFEN_ETIMEOUT if a bounded wait gave up; in both cases the
+ * outputs were left untouched.
  * ------------------------------------------------------------------------- */
+gefen_status_t gefen_refit_static_init(void);
 gefen_status_t gefen_refit_codebook_static(const float* x, int64_t n, const uint64_t* hist_in,
                                            int32_t bins, int32_t k, float* codebook_out,
                                            uint64_t* hist_out, int32_t* cell_start_out,
                                            double* cost_out, gefen_stream_t stream);
+gefen_status_t gefen_refit_static_status(int32_t* k_eff_out, gefen_stream_t stream);
 
 /* -------------------------------------------------------------------------
  * gefen_infer_blocks -- Algorithm 2 (Automatic Block Partitioning) for one

@@ -66,8 +66,6 @@ def _load():
     lib.oracle_step.argtypes = [i64, i64, P, P, P, P, P, P, P, i32, f64, f64,
                                 f64, f64, f64, i64, P, i32, i32]
     lib.oracle_step.restype = ctypes.c_int
-    lib.oracle_code_margin.argtypes = [f64, P, i32]
-    lib.oracle_code_margin.restype = f64
     lib.oracle_step_momentum.argtypes = [i64, i64, P, P, P, P, f64, P, P]
     lib.oracle_step_momentum.restype = ctypes.c_int
     lib.oracle_step_unquantized.argtypes = [i64, i64, P, P, P, P, f64, f64, f64,
@@ -114,11 +112,6 @@ def histogram(x: np.ndarray, bins: int, hist: np.ndarray | None = None) -> np.nd
 def nearest_level(x: float, codebook: np.ndarray) -> int:
     cb = np.ascontiguousarray(codebook, dtype=np.float32)
     return int(_load().oracle_nearest_level(float(x), _ptr(cb), cb.size))
-
-
-def code_margin(x: float, codebook: np.ndarray) -> float:
-    cb = np.ascontiguousarray(codebook, dtype=np.float32)
-    return float(_load().oracle_code_margin(float(x), _ptr(cb), cb.size))
 
 
 def step(theta, grad_bits, codes, v, s, cb_dec, cb_enc, *, period, lr, beta1,

@@ -179,20 +179,6 @@ int oracle_step(int64_t n, int64_t p, float* theta, const uint16_t* grad,
     return 0;
 }
 
-/* Decision margin of a code choice: (d2 - d1) / max(|x|, 2^-20), where d1 and
- * d2 are the distances from x to the nearest and second-nearest levels.  Used
- * by the parity tests to tell genuine disagreements from rounding flips. */
-double oracle_code_margin(double x, const float* C, int32_t k) {
-    double d1 = INFINITY, d2 = INFINITY;
-    for (int j = 0; j < k; ++j) {
-        double d = fabs(x - (double)C[j]);
-        if (d < d1) { d2 = d1; d1 = d; }
-        else if (d < d2) { d2 = d; }
-    }
-    double den = fabs(x) > ldexp(1.0, -20) ? fabs(x) : ldexp(1.0, -20);
-    return (d2 - d1) / den;
-}
-
 /* Momenta (unquantised) of one step, for margin checks: m_i as in
  * oracle_step, and s'_b.  Writes m (n doubles) and smax (n/p doubles). */
 int oracle_step_momentum(int64_t n, int64_t p, const uint16_t* grad,

@@ -27,6 +27,7 @@
 // canonical fp64 value once the final bound is known; their minimum, ties to
 // the smallest l, equals the full scan bit for bit.
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <mutex>
 
@@ -57,29 +58,36 @@ struct DpWs {
     double* D;     // (k+1) x (B+1)
     int32_t* A;    // (k+1) x (B+1)
     float2* E;     // (k+1) x (B+2): row kk, entry l = (hi, lo) of D[kk][l-1], read by level kk+1
-    uint32_t* sync;  // [0]: level-barrier arrivals; [kk]: next end position of level kk
+    int2* NS;      // B+1: near-optimal run starts [lo, hi] of each anchor row of the current level
+    uint32_t* sync;  // [0]: barrier arrivals; [1 + 3 kk + phase]: next row of level kk in that phase
 };
 
+// Counters: one barrier-arrival word, then three row counters per level.
+__host__ __device__ constexpr int sync_words(int k) { return 3 * (k + 1) + 2; }
+
 struct DpLayout {
-    size_t hdr, hist, idx, P0, P1, P2, D, A, E, sync, total;
+    size_t hdr, hist, idx, P0, P1, P2, D, A, E, NS, sync, total;
 };
+
+constexpr size_t cx_align(size_t x) { return (x + kWsAlign - 1) / kWsAlign * kWsAlign; }
 
 // Workspace: status header at offset 0 (so it can be read without knowing the
 // sizes), the histogram copy, then the DP arrays.
-DpLayout dp_layout(int B, int k) {
-    DpLayout L;
+constexpr DpLayout dp_layout(int B, int k) {
+    DpLayout L{};
     size_t o = 0;
     const size_t n1 = static_cast<size_t>(B) + 1;
-    L.hdr = o; o += align_up(sizeof(Header));
-    L.hist = o; o += align_up(static_cast<size_t>(B) * sizeof(uint64_t));
-    L.idx = o; o += align_up(n1 * sizeof(int32_t));
-    L.P0 = o;  o += align_up(n1 * sizeof(uint64_t));
-    L.P1 = o;  o += align_up(n1 * sizeof(int64_t));
-    L.P2 = o;  o += align_up(n1 * sizeof(uint64_t));
-    L.D = o;   o += align_up(static_cast<size_t>(k + 1) * n1 * sizeof(double));
-    L.A = o;   o += align_up(static_cast<size_t>(k + 1) * n1 * sizeof(int32_t));
-    L.E = o;   o += align_up(static_cast<size_t>(k + 1) * (n1 + 1) * sizeof(float2));
-    L.sync = o; o += align_up(static_cast<size_t>(k + 2) * sizeof(uint32_t));
+    L.hdr = o; o += cx_align(sizeof(Header));
+    L.hist = o; o += cx_align(static_cast<size_t>(B) * sizeof(uint64_t));
+    L.idx = o; o += cx_align(n1 * sizeof(int32_t));
+    L.P0 = o;  o += cx_align(n1 * sizeof(uint64_t));
+    L.P1 = o;  o += cx_align(n1 * sizeof(int64_t));
+    L.P2 = o;  o += cx_align(n1 * sizeof(uint64_t));
+    L.D = o;   o += cx_align(static_cast<size_t>(k + 1) * n1 * sizeof(double));
+    L.A = o;   o += cx_align(static_cast<size_t>(k + 1) * n1 * sizeof(int32_t));
+    L.E = o;   o += cx_align(static_cast<size_t>(k + 1) * (n1 + 1) * sizeof(float2));
+    L.NS = o;  o += cx_align(n1 * sizeof(int2));
+    L.sync = o; o += cx_align(static_cast<size_t>(sync_words(k)) * sizeof(uint32_t));
     L.total = o;
     return L;
 }
@@ -96,6 +104,7 @@ DpWs dp_ws(void* base, int B, int k) {
     w.D = reinterpret_cast<double*>(p + L.D);
     w.A = reinterpret_cast<int32_t*>(p + L.A);
     w.E = reinterpret_cast<float2*>(p + L.E);
+    w.NS = reinterpret_cast<int2*>(p + L.NS);
     w.sync = reinterpret_cast<uint32_t*>(p + L.sync);
     return w;
 }
@@ -185,18 +194,154 @@ __device__ __forceinline__ ff u128_to_ff(u128 v) {
                               __uint2float_rn(static_cast<uint32_t>(R)));
     return ff_quick(hi, r * __int_as_float((127 + e2) << 23));
 }
-__device__ __forceinline__ ff d_to_ff(double d) {
-    if (isinf(d)) return ff{static_cast<float>(d), 0.0f};
-    const float hi = __double2float_rn(d);
-    return ff{hi, __double2float_rn(__dsub_rn(d, static_cast<double>(hi)))};
+// ------------------------------------------- doubles handled as integer bits
+// Non-negative doubles order like their bit patterns, so the search converts,
+// compares and reduces them with integer operations: this part's fp64 pipe has
+// a small fraction of its integer and fp32 throughput.
+constexpr uint64_t kInfBits = 0x7FF0000000000000ull;
+
+__host__ __device__ __forceinline__ int clz64(uint64_t x) {  // x != 0
+#ifdef __CUDA_ARCH__
+    return __clzll(static_cast<long long>(x));
+#else
+    return __builtin_clzll(x);
+#endif
 }
+
+// Bits of the correctly rounded (to nearest, ties to even) double of an
+// unsigned 128-bit integer.
+__host__ __device__ __forceinline__ uint64_t u128_to_dbits(u128 v) {
+    int lz;
+    uint64_t top, rest;
+    if (v.hi) {
+        lz = clz64(v.hi);
+        top = lz ? (v.hi << lz) | (v.lo >> (64 - lz)) : v.hi;
+        rest = v.lo << lz;
+    } else if (v.lo) {
+        lz = 64 + clz64(v.lo);
+        top = v.lo << (lz - 64);
+        rest = 0;
+    } else {
+        return 0;
+    }
+    // value = top * 2^(64 - lz) with bit 63 of top set: keep 53 bits, round on
+    // the 11 below them and every bit of rest
+    uint64_t m = top >> 11;
+    const uint32_t g = static_cast<uint32_t>(top) & 0x7FFu;
+    m += (g > 0x400u || (g == 0x400u && (rest != 0 || (m & 1)))) ? 1 : 0;
+    int e = 127 - lz;  // exponent of the leading bit
+    if (m >> 53) {
+        m >>= 1;
+        ++e;
+    }
+    return (static_cast<uint64_t>(e + 1023) << 52) | (m & 0xFFFFFFFFFFFFFull);
+}
+
+constexpr uint64_t kMant = 0xFFFFFFFFFFFFFull;  // the 52 stored significand bits
+constexpr uint64_t kHidden = 1ull << 52;
+
+// Bits of RN(N / D) for positive normal doubles N, D (bits nb, db; N may be
+// +0) whose quotient is normal: the significand quotient by long division in
+// five 11-bit digits, each estimated in fp32 and corrected by one exact
+// integer step, then rounded to nearest (ties to even) with the remainder as
+// sticky bit.  Equal to IEEE division; integer and fp32 operations only.
+__host__ __device__ __forceinline__ uint64_t div_dbits(uint64_t nb, uint64_t db) {
+    if (nb == 0) return 0;
+    uint64_t Nm = (nb & kMant) | kHidden, Dm = (db & kMant) | kHidden;
+    int e = static_cast<int>(nb >> 52) - static_cast<int>(db >> 52);
+    if (Nm < Dm) {  // Nm / Dm in [1, 2) from here on
+        Nm <<= 1;
+        --e;
+    }
+    uint64_t R = Nm - Dm, Q = 1;
+#ifdef __CUDA_ARCH__
+    const float rd = __frcp_rn(__uint2float_rn(static_cast<uint32_t>(Dm >> 21)) * 2097152.0f);
+#else
+    const float rd = 1.0f / (static_cast<float>(static_cast<uint32_t>(Dm >> 21)) * 2097152.0f);
+#endif
+    for (int i = 0; i < 5; ++i) {
+        R <<= 11;  // R < Dm < 2^53 before the shift
+#ifdef __CUDA_ARCH__
+        const float rf = __uint2float_rn(static_cast<uint32_t>(R >> 32)) * 4294967296.0f;
+        uint64_t q = __float2uint_rz(rf * rd);
+#else
+        const float rf = static_cast<float>(static_cast<uint32_t>(R >> 32)) * 4294967296.0f;
+        uint64_t q = static_cast<uint64_t>(static_cast<uint32_t>(rf * rd));
+#endif
+        uint64_t p = q * Dm;  // q <= 2^11, so no overflow
+        if (p > R) {
+            --q;
+            p -= Dm;
+        }
+        R -= p;
+        if (R >= Dm) {
+            ++q;
+            R -= Dm;
+        }
+        Q = (Q << 11) | q;
+    }
+    // Q in [2^55, 2^56): 53 significand bits and three below them
+    uint64_t m = Q >> 3;
+    const uint32_t g = static_cast<uint32_t>(Q) & 7u;
+    m += (g > 4u || (g == 4u && (R != 0 || (m & 1)))) ? 1 : 0;
+    if (m >> 53) {
+        m >>= 1;
+        ++e;
+    }
+    return (static_cast<uint64_t>(e + 1023) << 52) | (m & kMant);
+}
+
+// Bits of RN(a + b) for non-negative normal (or zero) doubles a, b with a
+// finite sum: align with three extra bits (guard, round, sticky), add, round
+// to nearest (ties to even).  Equal to IEEE addition; integer operations only.
+__host__ __device__ __forceinline__ uint64_t add_dbits(uint64_t a, uint64_t b) {
+    if (a < b) {
+        const uint64_t t = a;
+        a = b;
+        b = t;
+    }
+    if (b == 0) return a;
+    int ea = static_cast<int>(a >> 52);
+    const int d = ea - static_cast<int>(b >> 52);
+    if (d > 54) return a;  // b below half an ulp of a
+    const uint64_t ma = ((a & kMant) | kHidden) << 3, mb = ((b & kMant) | kHidden) << 3;
+    uint64_t sm = ma + ((mb >> d) | (((mb & ((1ull << d) - 1)) != 0) ? 1 : 0));
+    if (sm >> 56) {
+        sm = (sm >> 1) | (sm & 1);
+        ++ea;
+    }
+    uint64_t m = sm >> 3;
+    const uint32_t g = static_cast<uint32_t>(sm) & 7u;
+    m += (g > 4u || (g == 4u && (m & 1))) ? 1 : 0;
+    if (m >> 53) {
+        m >>= 1;
+        ++ea;
+    }
+    return (static_cast<uint64_t>(ea) << 52) | (m & kMant);
+}
+
+// A non-negative double (bits) as a float-float value: hi holds its top 24
+// significant bits, lo the other 29 rounded once (relative error below
+// 2^-47).  DP values are 0, +inf, or at least 2^-62 (an integer numerator over
+// a count below 2^62) and below 2^127.
+__device__ __forceinline__ ff dbits_to_ff(uint64_t b) {
+    if (b >= kInfBits) return ff{INFINITY, 0.0f};
+    if (b == 0) return ff{0.0f, 0.0f};
+    const int e = static_cast<int>(b >> 52) - 1023;
+    const float hi = __uint_as_float((static_cast<uint32_t>(e + 127) << 23) | (static_cast<uint32_t>(b >> 29) & 0x7FFFFFu));
+    const float lo = __uint2float_rn(static_cast<uint32_t>(b) & 0x1FFFFFFFu) *
+                     __uint_as_float(static_cast<uint32_t>(e - 52 + 127) << 23);
+    return ff{hi, lo};
+}
+
 __device__ __forceinline__ ff cost_ff_interior(const Run& q) {
     return ff_div(u128_to_ff(interior_num(q.s0, q.s1, q.s2)), u128_to_ff(u128{0ull, q.s0}));
 }
 // Whether every value bounded below by lb is certainly above the best
-// screened value u (margin 2^-34 relative, far above the screening error).
-__device__ __forceinline__ bool excluded(ff lb, ff u) {
-    return ff_sub(lb, u).hi > kEps * (lb.hi + u.hi);
+// screened value u by more than da (margin 2^-34 relative, far above the
+// screening error, plus da).
+__device__ __forceinline__ bool excluded(ff lb, ff u, float da = 0.0f) {
+    return ff_sub(lb, u).hi > kEps * (lb.hi + u.hi) + da;
 }
 // Every level writes its own rows of D, A and E once, past L1, and they are
 // read only by later levels (after the grid barrier), so no SM can hold a stale
@@ -217,7 +362,7 @@ __global__ void __launch_bounds__(kPrefixThreads) k_dp_prefix(const uint64_t* __
     __shared__ int64_t s_p1[kPrefixThreads];
     __shared__ uint64_t s_hi[kPrefixThreads];
     const int t = threadIdx.x;
-    if (t < k + 2) W.sync[t] = 0u;
+    if (t < sync_words(k)) W.sync[t] = 0u;
     const int per = (B + kPrefixThreads - 1) / kPrefixThreads;
     const int i0 = min(B, t * per), i1 = min(B, i0 + per);
     uint64_t cnt = 0, p0 = 0, p2 = 0, hi = 0;
@@ -299,25 +444,23 @@ __global__ void __launch_bounds__(kDpThreads) k_dp_level1(int B, DpWs W) {
         W.D[r] = (r == 0) ? 0.0 : INFINITY;
         W.A[r] = 0;
     }
-    double d = INFINITY;
-    if (r >= 1 && r <= h.b) {
-        d = u128_to_double_rn(fixed_num(W.P0[r], W.P1[r], W.P2[r], B, +1));
-    }
+    uint64_t d = kInfBits;
+    if (r >= 1 && r <= h.b) d = u128_to_dbits(fixed_num(W.P0[r], W.P1[r], W.P2[r], B, +1));
     if (r >= 0) {
-        W.D[n1 + r] = d;
+        W.D[n1 + r] = __longlong_as_double(static_cast<long long>(d));
         W.A[n1 + r] = (r >= 1 && r <= h.b) ? 1 : 0;
     }
-    const ff e = d_to_ff(d);
+    const ff e = dbits_to_ff(d);
     W.E[1 * (n1 + 1) + g] = make_float2(e.hi, e.lo);  // row 1 of E
 }
 
-// Candidate screen + canonical evaluation for one (r, level) -- interior.
+// Candidate screen + canonical evaluation for one (r, level).
 struct Best {
-    double v;
+    uint64_t v;  // bits of a non-negative double
     int l;
 };
 
-__device__ __forceinline__ void take(Best& b, double v, int l) {
+__device__ __forceinline__ void take(Best& b, uint64_t v, int l) {
     if (v < b.v || (v == b.v && l < b.l)) { b.v = v; b.l = l; }
 }
 
@@ -334,14 +477,13 @@ __device__ __forceinline__ ff warp_min_ff(ff v) {
     const int lk = __reduce_min_sync(0xffffffffu, hb == hm ? lo_key(v.lo) : 0x7FFFFFFF);
     return ff{__uint_as_float(hm), __int_as_float(lk >= 0 ? lk : (lk ^ 0x7FFFFFFF))};
 }
+// Lexicographic (value, l) minimum over the warp: three integer reductions.
 __device__ __forceinline__ Best warp_min_best(Best b) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        const double ov = __shfl_xor_sync(0xffffffffu, b.v, o);
-        const int ol = __shfl_xor_sync(0xffffffffu, b.l, o);
-        take(b, ov, ol);
-    }
-    return b;
+    const unsigned h = static_cast<unsigned>(b.v >> 32), lo = static_cast<unsigned>(b.v);
+    const unsigned hm = __reduce_min_sync(0xffffffffu, h);
+    const unsigned lm = __reduce_min_sync(0xffffffffu, h == hm ? lo : 0xFFFFFFFFu);
+    const unsigned l = __reduce_min_sync(0xffffffffu, (h == hm && lo == lm) ? static_cast<unsigned>(b.l) : 0x7FFFFFFFu);
+    return Best{(static_cast<uint64_t>(hm) << 32) | lm, static_cast<int>(l)};
 }
 
 constexpr int kDpWarps = 16;     // warps (end positions at a time) per CTA
@@ -364,14 +506,17 @@ __device__ __forceinline__ ff run_cost_ff(const RowCtx& c, int l) {
     return c.last ? u128_to_ff(fixed_num(q.s0, q.s1, q.s2, c.B, -1)) : cost_ff_interior(q);
 }
 
-// Canonical value of candidate l: D[l-1] + cost(l..r), each rounded as the
-// oracle rounds them (fp64; slow on this part, so used only for near-ties).
-__device__ __forceinline__ double canonical(const RowCtx& c, int l) {
+// Canonical value of candidate l (bits): D[l-1] + cost(l..r), each rounded
+// as the oracle rounds them -- the conversions, the division and the sum in
+// integer arithmetic that reproduces IEEE round-to-nearest (this part's fp64
+// pipe is slow).  Used only for candidates near the minimum.
+__device__ __forceinline__ uint64_t canonical(const RowCtx& c, int l) {
     const Run q = run_of(*c.W, l, c.P0r, c.P1r, c.P2r);
-    const double dprev = __ldca(c.Dp + l - 1);
-    const double cost = c.last ? u128_to_double_rn(fixed_num(q.s0, q.s1, q.s2, c.B, -1))
-                               : __ddiv_rn(u128_to_double_rn(interior_num(q.s0, q.s1, q.s2)), __ull2double_rn(q.s0));
-    return __dadd_rn(dprev, cost);
+    const uint64_t dprev = __ldca(reinterpret_cast<const unsigned long long*>(c.Dp) + l - 1);
+    const uint64_t cost = c.last ? u128_to_dbits(fixed_num(q.s0, q.s1, q.s2, c.B, -1))
+                                 : div_dbits(u128_to_dbits(interior_num(q.s0, q.s1, q.s2)),
+                                             u128_to_dbits(u128{0ull, q.s0}));
+    return add_dbits(dprev, cost);
 }
 
 // Search state of one warp: u is the best screened value seen; each lane
@@ -380,15 +525,35 @@ __device__ __forceinline__ double canonical(const RowCtx& c, int l) {
 // it.  A second pending candidate in the same lane first settles the first.
 // Every candidate the final u does not exclude thus gets its canonical value,
 // and the best of those is the full scan's.
+//
+// An anchor row also records the extent [nlo, nhi] of its near-optimal
+// candidates: every l whose exact value is within da of the row minimum (runs
+// and candidates are then excluded only beyond the relative margin plus da).
 struct Search {
     ff u;
     int pl;  // pending candidate of this lane, 0 if none
     ff pv;   // its screened value
     Best bst;
+    float da;      // absolute margin of the near-optimal extent (0: not recorded)
+    int nlo, nhi;  // extent of the near-optimal candidates this lane settled
 };
 
+__device__ __forceinline__ void search_init(Search& S, float da) {
+    S.u = ff{INFINITY, 0.0f};
+    S.pl = 0;
+    S.pv = ff{INFINITY, 0.0f};
+    S.bst = Best{kInfBits, 0};
+    S.da = da;
+    S.nlo = 0x7FFFFFFF;
+    S.nhi = 0;
+}
+
 __device__ __forceinline__ void settle(const RowCtx& c, Search& S) {
-    if (S.pl != 0 && !excluded(S.pv, S.u)) take(S.bst, canonical(c, S.pl), S.pl);
+    if (S.pl != 0 && !excluded(S.pv, S.u, S.da)) {
+        S.nlo = min(S.nlo, S.pl);
+        S.nhi = max(S.nhi, S.pl);
+        if (!excluded(S.pv, S.u)) take(S.bst, canonical(c, S.pl), S.pl);
+    }
     S.pl = 0;
 }
 
@@ -400,7 +565,7 @@ __device__ __forceinline__ void eval_lanes(const RowCtx& c, int l, Search& S) {
     if (in) v = ff_add(ld_ff(c.Ep, l), run_cost_ff(c, l));
     const ff vm = warp_min_ff(v);
     if (vm.hi < S.u.hi || (vm.hi == S.u.hi && vm.lo < S.u.lo)) S.u = vm;
-    if (in && !excluded(v, S.u)) {
+    if (in && !excluded(v, S.u, S.da)) {
         settle(c, S);
         S.pl = l;
         S.pv = v;
@@ -412,31 +577,28 @@ __device__ __forceinline__ void eval_candidates(const RowCtx& c, int a, int e, i
     eval_lanes(c, l <= e ? l : 0, S);
 }
 
-__device__ Best search_row(const RowCtx& c, int kk, int hint, int lane, int2* stack) {
-    Search S;
-    S.u = ff{INFINITY, 0.0f};
-    S.pl = 0;
-    S.pv = ff{INFINITY, 0.0f};
-    S.bst = Best{INFINITY, 0};
-    const int r = c.r;
-    if (kk == 2 && r - kk >= 64) {
+// Every candidate l in [lo, hi] of one row, pruned: a 32-wide window around
+// the hint, then the rest by 32-way subdivision.  Leaves the result in S.
+__device__ void search_row(const RowCtx& c, int kk, int lo, int hi, int hint, int lane, int2* stack, Search& S) {
+    if (kk == 2 && hi - lo >= 64) {
         // level 2: the previous level's split (always 1) says nothing, so
         // sample 32 evenly spaced candidates and centre the window on the best
-        const int st = (r - kk) / 31;
-        eval_candidates(c, kk, r, lane, S, st);
+        const int st = (hi - lo) / 31;
+        eval_candidates(c, lo, hi, lane, S, st);
         const unsigned at = __ballot_sync(0xffffffffu, S.pl != 0 && S.pv.hi == S.u.hi && S.pv.lo == S.u.lo);
-        hint = at ? __shfl_sync(0xffffffffu, S.pl, __ffs(at) - 1) : kk + (r - kk) / 2;
+        hint = at ? __shfl_sync(0xffffffffu, S.pl, __ffs(at) - 1) : lo + (hi - lo) / 2;
     }
-    int w0 = max(kk, hint - 8);
-    const int w1 = min(r, w0 + 31);
-    w0 = max(kk, w1 - 31);
+    hint = min(max(hint, lo), hi);
+    int w0 = max(lo, hint - 8);
+    const int w1 = min(hi, w0 + 31);
+    w0 = max(lo, w1 - 31);
     eval_candidates(c, w0, w1, lane, S);
     int sp = 0;  // warp-uniform
     if (lane == 0) {
-        if (w1 < r) stack[sp] = make_int2(w1 + 1, r);
-        if (w0 > kk) stack[sp + (w1 < r ? 1 : 0)] = make_int2(kk, w0 - 1);
+        if (w1 < hi) stack[sp] = make_int2(w1 + 1, hi);
+        if (w0 > lo) stack[sp + (w1 < hi ? 1 : 0)] = make_int2(lo, w0 - 1);
     }
-    sp = (w1 < r ? 1 : 0) + (w0 > kk ? 1 : 0);
+    sp = (w1 < hi ? 1 : 0) + (w0 > lo ? 1 : 0);
     __syncwarp();
     while (sp > 0) {
         if (stack[sp - 1].y - stack[sp - 1].x < 32) {
@@ -462,7 +624,7 @@ __device__ Best search_row(const RowCtx& c, int kk, int hint, int lane, int2* st
         const int cw = (width + 31) >> 5;
         const int ca = a + lane * cw, ce = min(e, ca + cw - 1);
         bool keep = false;
-        if (ca <= e) keep = !excluded(ff_add(ld_ff(c.Ep, ca), run_cost_ff(c, ce)), S.u);
+        if (ca <= e) keep = !excluded(ff_add(ld_ff(c.Ep, ca), run_cost_ff(c, ce)), S.u, S.da);
         const unsigned mask = __ballot_sync(0xffffffffu, keep);
         const int cnt = __popc(mask);
         if (sp + cnt > kStackCap) {
@@ -478,18 +640,35 @@ __device__ Best search_row(const RowCtx& c, int kk, int hint, int lane, int2* st
         __syncwarp();
     }
     settle(c, S);
-    return warp_min_best(S.bst);
 }
 
-// Level kk at end position r: interior (2 <= kk < k_eff) for every r, or the
-// last level (kk == k_eff) for r = b only, or nothing defined (kk > k_eff).
-// Every D[kk][r] is written (+inf where undefined).
-__device__ __forceinline__ void level_row(int B, int kk, int r, const DpWs& W, const Header& h, int lane,
-                                          int2* stack) {
+// How a row of a level is searched.
+enum RowMode {
+    kRowFull = 0,     // every run start in [kk, r]
+    kRowAnchor = 1,   // the same, recording the near-optimal extent in NS[r]
+    kRowBracket = 2,  // only the run starts between the extents of the two nearest anchors
+};
+
+// Anchored bracketing.  With V(r, l) = D[kk-1][l-1] + cost(l..r) in exact
+// arithmetic, the interior cost satisfies the quadrangle inequality
+// cost(a..c) + cost(b..d) <= cost(a..d) + cost(b..c) for a <= b <= c <= d (the
+// squared error of contiguous cells of points on a line), and the D terms
+// cancel, so for r1 < r2 and l < l':  V(r1,l) + V(r2,l') <= V(r1,l') + V(r2,l).
+// Take an anchor row a < r and a minimiser l* of row a.  For l < l*:
+// V(r,l) - V(r,l*) >= V(a,l) - V(a,l*), so every l below the anchor's
+// near-optimal extent (V(a,l) > min_a + da) has V(r,l) > min_r + da; likewise,
+// with an anchor a' > r, every l above its extent.  da is 2^-39 of the largest
+// D[kk-1][x] over the rows the anchor serves, and min_r <= D[kk-1][r-1] (the
+// run [r..r] costs 0), so da exceeds 2^9 times the rounding of the canonical
+// fp64 values (under 2^-49 relative): no run start outside the bracket can
+// win or tie the canonical minimum, and the bracketed rows give the full
+// scan's result bit for bit.
+__device__ void level_row(int B, int kk, int r, int stride, int mode, const DpWs& W, const Header& h, int lane,
+                          int2* stack) {
     const int n1 = B + 1;
     const bool last = (kk == h.k_eff);
     const bool active = kk <= h.k_eff && r <= h.b && (last ? (r == h.b) : (r >= kk));
-    double d = INFINITY;
+    uint64_t d = kInfBits;
     int al = 0;
     if (active) {
         RowCtx c;
@@ -502,36 +681,104 @@ __device__ __forceinline__ void level_row(int B, int kk, int r, const DpWs& W, c
         c.B = B;
         c.r = r;
         c.last = last;
+        float da = 0.0f;
+        int lo = kk, hi = r;
+        if (mode == kRowAnchor) {
+            // rows served: (r - stride, r + stride), whose minima are at most
+            // D[kk-1][x] for x in [r - stride, r + stride - 2]
+            float dm = 0.0f;
+            const int x0 = max(kk - 1, r - stride), x1 = min(h.b, r + stride - 2);
+            for (int x = x0 + lane; x <= x1; x += 32) dm = fmaxf(dm, __ldca(&c.Ep[x + 1].x));
+            dm = __uint_as_float(__reduce_max_sync(0xffffffffu, __float_as_uint(dm)));  // dm >= 0
+            da = dm * 0x1p-39f;
+        } else if (mode == kRowBracket) {
+            const int a1 = (r / stride) * stride, a2 = min(a1 + stride, h.b);
+            if (a1 >= kk) lo = max(lo, __ldcg(W.NS + a1).x);
+            hi = min(hi, __ldcg(W.NS + a2).y);
+            if (lo > hi) { lo = kk; hi = r; }  // never expected: the whole range
+        }
         // hint: the previous level's split at r, moved by its share of the last cell
         const int hp = max(kk, __ldca(W.A + static_cast<size_t>(kk - 1) * n1 + r));
         const int hint = hp + (r - hp) / kk;
-        const Best b = search_row(c, kk, hint, lane, stack);
+        Search S;
+        search_init(S, da);
+        search_row(c, kk, lo, hi, hint, lane, stack, S);
+        const Best b = warp_min_best(S.bst);
         d = b.v;
         al = b.l;
+        if (mode == kRowAnchor) {
+            const int nlo = __reduce_min_sync(0xffffffffu, S.nlo);
+            const int nhi = __reduce_max_sync(0xffffffffu, S.nhi);
+            if (lane == 0) __stcg(W.NS + r, make_int2(nlo, nhi));
+        }
     }
     if (lane == 0) {
         // stored past L1 (.cg): no SM may cache part of a row before the level ends
-        __stcg(W.D + static_cast<size_t>(kk) * n1 + r, d);
+        __stcg(reinterpret_cast<unsigned long long*>(W.D) + static_cast<size_t>(kk) * n1 + r,
+               static_cast<unsigned long long>(d));
         __stcg(W.A + static_cast<size_t>(kk) * n1 + r, al);
-        const ff e = d_to_ff(d);
+        const ff e = dbits_to_ff(d);
         float2* En = W.E + static_cast<size_t>(kk) * (n1 + 1);
         __stcg(En + r + 1, make_float2(e.hi, e.lo));
         if (r == 0) __stcg(En, make_float2(INFINITY, 0.0f));
     }
 }
 
-__device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
+__device__ __forceinline__ uint32_t ld_acquire(const void* p) {
     uint32_t v;
     asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     return v;
 }
 
-// Levels 2..k in one cooperative launch (every CTA resident).  Warp w of the
-// grid takes end position w of each level, and positions past the grid's
-// warps come from a counter; a grid barrier separates the levels.  The
-// barrier's wait gives up after about a second (status 2), so a lost CTA
-// cannot hang the GPU.
-__global__ void __launch_bounds__(kDpWarps * 32) k_dp_levels(int B, int k, DpWs W) {
+struct DpLaunch {
+    int B, k;
+    int stride;              // anchor spacing; 0: every row searched over its whole range
+    uint32_t barrier_extra;  // added to every barrier target (0; a test hook makes it unreachable)
+    long long spin;          // cycles a barrier wait may take before it gives up
+};
+
+// Grid barrier of the cooperative launch.  The wait gives up after P.spin
+// cycles, or as soon as another CTA has given up (status 2), so a lost CTA
+// cannot hang the GPU.  Returns true when the CTA must stop.
+__device__ __forceinline__ bool grid_barrier(const DpWs& W, uint32_t target, long long spin, int* s_abort) {
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();  // this CTA's rows before its arrival
+        atomicAdd(W.sync, 1u);
+        const long long t0 = clock64();
+        int ab = 0;
+        while (ld_acquire(W.sync) < target) {
+            if (ld_acquire(&W.hdr->status) != 0u || clock64() - t0 > spin) {
+                ab = 1;
+                atomicCAS(&W.hdr->status, 0, 2);
+                break;
+            }
+        }
+        *s_abort = ab;
+    }
+    __syncthreads();
+    return *s_abort != 0;
+}
+
+// Rows 0..n-1 of one phase over the grid's warps: warp gw takes row gw, the
+// rest come from the phase's counter.
+template <class F>
+__device__ __forceinline__ void for_rows(int n, uint32_t* counter, int gw, int nwarps, int lane, F&& f) {
+    int i = gw;
+    while (i < n) {
+        f(i);
+        if (nwarps >= n) break;
+        int ni = 0;
+        if (lane == 0) ni = nwarps + static_cast<int>(atomicAdd(counter, 1u));
+        i = __shfl_sync(0xffffffffu, ni, 0);
+    }
+}
+
+// Levels 2..k in one cooperative launch (every CTA resident), a grid barrier
+// between levels.  With anchors (P.stride > 0, interior levels), a level runs
+// in two phases: the anchor rows r = 0, stride, 2 stride, ... and b, then
+// (after a barrier) every other row, bracketed by its two anchors.
+__global__ void __launch_bounds__(kDpWarps * 32) k_dp_levels(DpLaunch P, DpWs W) {
     __shared__ int2 s_stack[kDpWarps][kStackCap];
     __shared__ int s_abort;
     const Header h = *W.hdr;
@@ -539,34 +786,27 @@ __global__ void __launch_bounds__(kDpWarps * 32) k_dp_levels(int B, int k, DpWs 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t G = gridDim.x;
     const int nwarps = static_cast<int>(G) * kDpWarps;
-    for (int kk = 2; kk <= k; ++kk) {
-        int r = static_cast<int>(blockIdx.x) * kDpWarps + warp;
-        while (r <= B) {
-            level_row(B, kk, r, W, h, lane, s_stack[warp]);
-            if (nwarps > B) break;  // every position had a warp of its own
-            int nr = 0;
-            if (lane == 0) nr = nwarps + static_cast<int>(atomicAdd(W.sync + kk, 1u));
-            r = __shfl_sync(0xffffffffu, nr, 0);
+    const int gw = static_cast<int>(blockIdx.x) * kDpWarps + warp;
+    const int B = P.B, S = P.stride;
+    int2* stack = s_stack[warp];
+    uint32_t nbar = 0;
+    for (int kk = 2; kk <= P.k; ++kk) {
+        uint32_t* ctr = W.sync + 1 + 3 * kk;
+        if (S > 0 && kk < h.k_eff && h.b > S) {
+            const int nA = h.b / S + 1 + (h.b % S ? 1 : 0);
+            for_rows(nA, ctr + 1, gw, nwarps, lane,
+                     [&](int i) { level_row(B, kk, min(i * S, h.b), S, kRowAnchor, W, h, lane, stack); });
+            if (grid_barrier(W, ++nbar * G + P.barrier_extra, P.spin, &s_abort)) return;
+            for_rows(B + 1, ctr + 2, gw, nwarps, lane, [&](int r) {
+                if (r <= h.b && (r % S == 0 || r == h.b)) return;  // an anchor
+                level_row(B, kk, r, S, kRowBracket, W, h, lane, stack);
+            });
+        } else {
+            for_rows(B + 1, ctr, gw, nwarps, lane,
+                     [&](int r) { level_row(B, kk, r, S, kRowFull, W, h, lane, stack); });
         }
-        if (kk == k) break;
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            __threadfence();  // this CTA's rows of level kk before its arrival
-            atomicAdd(W.sync, 1u);
-            const uint32_t target = static_cast<uint32_t>(kk - 1) * G;
-            const long long t0 = clock64();
-            int ab = 0;
-            while (ld_acquire(W.sync) < target) {
-                if (clock64() - t0 > (1ll << 31)) {
-                    ab = 1;
-                    atomicExch(&W.hdr->status, 2);
-                    break;
-                }
-            }
-            s_abort = ab;
-        }
-        __syncthreads();
-        if (s_abort) return;
+        if (kk == P.k) break;
+        if (grid_barrier(W, ++nbar * G + P.barrier_extra, P.spin, &s_abort)) return;
     }
 }
 
@@ -636,6 +876,37 @@ __global__ void k_dp_backtrack(int B, int k, DpWs W, float* __restrict__ codeboo
 
 using namespace gefen;
 
+namespace {
+
+constexpr int kAnchorStride = 16;           // rows between anchors (automatic choice)
+constexpr long long kBarrierSpin = 1ll << 31;  // about a second at the SM clock
+
+// Test hooks (gefen_refit_debug): anchor stride (-1 automatic), barrier target
+// offset, barrier wait limit (0: kBarrierSpin).
+std::atomic<int> g_dbg_stride{-1};
+std::atomic<uint32_t> g_dbg_barrier_extra{0};
+std::atomic<long long> g_dbg_spin{0};
+
+// Resident CTAs per SM of k_dp_levels, asked once per device.
+int dp_levels_per_sm() {
+    static std::mutex mu;
+    static int cached[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+    std::lock_guard<std::mutex> g(mu);
+    if (cached[dev] == 0) {
+        int n = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_dp_levels, kDpWarps * 32, 0) != cudaSuccess) {
+            (void)cudaGetLastError();
+            return 0;
+        }
+        cached[dev] = n;
+    }
+    return cached[dev];
+}
+
+}  // namespace
+
 extern "C" size_t gefen_refit_workspace_size(int32_t bins, int32_t k) {
     if (bins < 1 || bins > GEFEN_MAX_BINS || k < 2 || k > GEFEN_MAX_LEVELS) return 0;
     return dp_layout(bins, k).total;
@@ -675,15 +946,23 @@ extern "C" gefen_status_t gefen_refit_codebook(const float* x, int64_t n, const 
     const int grid1 = (bins + 2 + kDpThreads - 1) / kDpThreads;
     k_dp_level1<<<grid1, kDpThreads, 0, st>>>(bins, W);
     {
-        static int per_sm = 0;  // resident CTAs per SM (a property of the kernel)
-        if (per_sm == 0 &&
-            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_dp_levels, kDpWarps * 32, 0) != cudaSuccess)
-            return GEFEN_ECUDA;
+        const int per_sm = dp_levels_per_sm();
+        if (per_sm < 1) return GEFEN_ECUDA;
         const int rows = (bins + 1 + kDpWarps - 1) / kDpWarps;  // CTAs with a row each
-        int grid = std::max(1, std::min(per_sm * device_sm_count(), rows));
-        int bb = bins, kv = k;
+        const int grid = std::max(1, std::min(per_sm * device_sm_count(), rows));
+        DpLaunch P;
+        P.B = bins;
+        P.k = k;
+        // anchors pay off once the rows outnumber the grid's warps: each warp
+        // then searches one anchor row in full and brackets the rest
+        const int auto_stride = (bins + 1 > 2 * grid * kDpWarps) ? kAnchorStride : 0;
+        const int forced = g_dbg_stride.load();
+        P.stride = forced >= 0 ? forced : auto_stride;
+        P.barrier_extra = g_dbg_barrier_extra.load();
+        const long long spin = g_dbg_spin.load();
+        P.spin = spin > 0 ? spin : kBarrierSpin;
         DpWs w = W;
-        void* args[] = {&bb, &kv, &w};
+        void* args[] = {&P, &w};
         if (cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(k_dp_levels), dim3(grid), dim3(kDpWarps * 32),
                                         args, 0, st) != cudaSuccess)
             return GEFEN_ECUDA;
@@ -731,15 +1010,7 @@ namespace {
 constexpr int kStaticMaxBins = 4096;
 constexpr int kStaticMaxLevels = 256;
 
-constexpr size_t cx_align(size_t x) { return (x + kWsAlign - 1) / kWsAlign * kWsAlign; }
-// Mirrors dp_layout(kStaticMaxBins, kStaticMaxLevels).
-constexpr size_t kStaticScratchBytes =
-    cx_align(sizeof(Header)) + cx_align(size_t(kStaticMaxBins) * sizeof(uint64_t)) +
-    cx_align(size_t(kStaticMaxBins + 1) * sizeof(int32_t)) + 3 * cx_align(size_t(kStaticMaxBins + 1) * 8) +
-    cx_align(size_t(kStaticMaxLevels + 1) * (kStaticMaxBins + 1) * sizeof(double)) +
-    cx_align(size_t(kStaticMaxLevels + 1) * (kStaticMaxBins + 1) * sizeof(int32_t)) +
-    cx_align(size_t(kStaticMaxLevels + 1) * (kStaticMaxBins + 2) * sizeof(float2)) +
-    cx_align(size_t(kStaticMaxLevels + 2) * sizeof(uint32_t));
+constexpr size_t kStaticScratchBytes = dp_layout(kStaticMaxBins, kStaticMaxLevels).total;
 
 __device__ __align__(256) unsigned char g_refit_scratch[kStaticScratchBytes];
 
@@ -753,7 +1024,21 @@ gefen_status_t static_scratch(void** out) {
     std::lock_guard<std::mutex> g(g_scratch_mu);
     if (g_scratch_addr[dev] == nullptr) {
         void* p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_refit_scratch) != cudaSuccess || p == nullptr) return GEFEN_ECUDA;
+        if (cudaGetSymbolAddress(&p, g_refit_scratch) != cudaSuccess || p == nullptr) {
+            (void)cudaGetLastError();
+            return GEFEN_ECUDA;
+        }
+        // load the refit's kernels now as well, so that a later call needs
+        // nothing more from the driver
+        cudaFuncAttributes fa;
+        if (cudaFuncGetAttributes(&fa, k_dp_prefix) != cudaSuccess ||
+            cudaFuncGetAttributes(&fa, k_dp_level1) != cudaSuccess ||
+            cudaFuncGetAttributes(&fa, k_dp_levels) != cudaSuccess ||
+            cudaFuncGetAttributes(&fa, k_dp_backtrack) != cudaSuccess || dp_levels_per_sm() < 1 ||
+            prepare_histogram() != cudaSuccess) {
+            (void)cudaGetLastError();
+            return GEFEN_ECUDA;
+        }
         g_scratch_addr[dev] = p;
     }
     *out = g_scratch_addr[dev];
@@ -761,6 +1046,12 @@ gefen_status_t static_scratch(void** out) {
 }
 
 }  // namespace
+
+extern "C" gefen_status_t gefen_refit_static_init(void) {
+    if (gefen_status_t s = check_device(); s != GEFEN_OK) return s;
+    void* scratch = nullptr;
+    return static_scratch(&scratch);
+}
 
 extern "C" gefen_status_t gefen_refit_codebook_static(const float* x, int64_t n, const uint64_t* hist_in,
                                                       int32_t bins, int32_t k, float* codebook_out,
@@ -773,4 +1064,19 @@ extern "C" gefen_status_t gefen_refit_codebook_static(const float* x, int64_t n,
     if (gefen_status_t s = static_scratch(&scratch); s != GEFEN_OK) return s;
     return gefen_refit_codebook(x, n, hist_in, bins, k, codebook_out, hist_out, cell_start_out, cost_out, scratch,
                                 kStaticScratchBytes, stream);
+}
+
+extern "C" gefen_status_t gefen_refit_static_status(int32_t* k_eff_out, gefen_stream_t stream) {
+    void* scratch = nullptr;
+    if (gefen_status_t s = static_scratch(&scratch); s != GEFEN_OK) return s;
+    return gefen_refit_status(scratch, k_eff_out, stream);
+}
+
+extern "C" gefen_status_t gefen_refit_debug(int32_t anchor_stride, uint32_t barrier_extra,
+                                            int64_t barrier_spin_cycles) {
+    if (anchor_stride < -1 || anchor_stride > GEFEN_MAX_BINS || barrier_spin_cycles < 0) return GEFEN_EINVAL;
+    g_dbg_stride.store(anchor_stride);
+    g_dbg_barrier_extra.store(barrier_extra);
+    g_dbg_spin.store(barrier_spin_cycles);
+    return GEFEN_OK;
 }

@@ -156,6 +156,13 @@ __global__ void __launch_bounds__(kHistThreads) k_hist16(const float* __restrict
 
 }  // namespace
 
+cudaError_t prepare_histogram() {
+    cudaFuncAttributes fa;
+    cudaError_t e = cudaFuncGetAttributes(&fa, k_hist1);
+    if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, k_hist16);
+    return e;
+}
+
 cudaError_t launch_histogram(const float* x, const HistRange* ranges, int nranges, int bins, uint64_t* hist,
                              cudaStream_t stream) {
     // One launch sees at most 2^36 values, so a CTA's u32 counters (it handles

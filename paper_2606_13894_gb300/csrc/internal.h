@@ -23,6 +23,10 @@ struct HistRange {
 cudaError_t launch_histogram(const float* x, const HistRange* ranges, int nranges,
                              int bins, uint64_t* hist, cudaStream_t stream);
 
+// Loads the histogram kernels on the current device (so that a later launch
+// needs nothing more from the driver).
+cudaError_t prepare_histogram();
+
 // Multiprocessor count of the current device (cached per device).
 int device_sm_count();
 

@@ -48,7 +48,8 @@ EXPORTS = ("gefen_status_string", "gefen_sync_status", "gefen_step_workspace_siz
            "gefen_step_status",
            "gefen_refit_workspace_size", "gefen_refit_codebook", "gefen_refit_status",
            "gefen_refit_tables", "gefen_infer_workspace_size", "gefen_infer_blocks",
-           "gefen_refit_codebook_static", "gefen_muon_workspace_size", "gefen_muon_step")
+           "gefen_refit_codebook_static", "gefen_refit_static_init", "gefen_refit_static_status",
+           "gefen_refit_debug", "gefen_muon_workspace_size", "gefen_muon_step")
 
 GEFEN_MUON_BF16_GEMM = 1
 
@@ -95,6 +96,12 @@ def load(build_if_needed: bool = True):
         L.gefen_refit_codebook.restype = ctypes.c_int
         L.gefen_refit_codebook_static.argtypes = [P, i64, P, i32, i32, P, P, P, P, P]
         L.gefen_refit_codebook_static.restype = ctypes.c_int
+        L.gefen_refit_static_init.argtypes = []
+        L.gefen_refit_static_init.restype = ctypes.c_int
+        L.gefen_refit_static_status.argtypes = [ctypes.POINTER(i32), P]
+        L.gefen_refit_static_status.restype = ctypes.c_int
+        L.gefen_refit_debug.argtypes = [i32, ctypes.c_uint32, i64]
+        L.gefen_refit_debug.restype = ctypes.c_int
         L.gefen_refit_status.argtypes = [P, ctypes.POINTER(i32), P]
         L.gefen_refit_status.restype = ctypes.c_int
         L.gefen_refit_tables.argtypes = [P, i32, i32, P, P, P]
@@ -230,6 +237,25 @@ def gefen_refit_codebook_static(*, bins: int, k: int, codebook_out, x=None, hist
     st = load().gefen_refit_codebook_static(xp, n, _ptr(hist_in), bins, k, _ptr(codebook_out), _ptr(hist_out),
                                             _ptr(cell_start_out), _ptr(cost_out), _stream(stream))
     _check("gefen_refit_codebook_static", st)
+
+
+def gefen_refit_static_init():
+    """Loads the static refit's module, array and kernels on the current device."""
+    _check("gefen_refit_static_init", load().gefen_refit_static_init())
+
+
+def gefen_refit_static_status(stream=None) -> int:
+    """Status of the last static refit on the current device (waits for the
+    stream); raises on a device-side failure; returns k_eff."""
+    ke = ctypes.c_int32(0)
+    _check("gefen_refit_static_status", load().gefen_refit_static_status(ctypes.byref(ke), _stream(stream)))
+    return int(ke.value)
+
+
+def gefen_refit_debug(anchor_stride: int = -1, barrier_extra: int = 0, barrier_spin_cycles: int = 0):
+    """Test hook of the refit (see gefen.h); (-1, 0, 0) restores the defaults."""
+    _check("gefen_refit_debug", load().gefen_refit_debug(int(anchor_stride), int(barrier_extra),
+                                                         int(barrier_spin_cycles)))
 
 
 def gefen_refit_status(workspace_buf, stream=None) -> int:

@@ -1,6 +1,11 @@
 """Host-side checks of the C ABI: the library builds and loads, exports every
 function include/gefen.h declares, and rejects bad arguments on the host
-(before any device work), so none of these calls needs a GPU."""
+(before any device work), so none of these calls needs a GPU.
+
+The calls pass fake device pointers and rely on the host-side validation
+returning first.  They run only in a process that sees no CUDA device
+(tests/test_abi_host_isolated.py starts one), so that a validation regression
+ends in the library's device check instead of a launch on a bogus address."""
 import ctypes
 import os
 import re
@@ -8,6 +13,9 @@ import re
 import pytest
 
 from paper_2606_13894_gb300 import gefen as G
+
+pytestmark = pytest.mark.skipif(os.environ.get("CUDA_VISIBLE_DEVICES") != "",
+                                reason="runs in a child process with no visible CUDA device")
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 HEADER = os.path.join(ROOT, "include", "gefen.h")

@@ -75,9 +75,20 @@ def _t_hist(B, n, seed):
     return oracle.histogram(x, B)
 
 
+@pytest.fixture
+def anchor_stride(request):
+    """Forces the DP's anchor stride for one test (0: every end position
+    searched over its whole range; s: an anchor every s positions, the other
+    positions bracketed by their two anchors), then restores the default."""
+    G.gefen_refit_debug(request.param, 0, 0)
+    yield request.param
+    G.gefen_refit_debug(-1, 0, 0)
+
+
+@pytest.mark.parametrize("anchor_stride", [0, 2, 7, 32], indirect=True)
 @pytest.mark.parametrize("B,k,kind", [(64, 3, "rand"), (512, 16, "rand"), (4096, 256, "t"), (1024, 256, "rand"),
-                                      (4096, 16, "t"), (300, 2, "rand"), (65536, 4, "rand")])
-def test_dp_bit_exact_with_full_tables(B, k, kind):
+                                      (4096, 16, "t"), (300, 2, "rand"), (65536, 4, "rand"), (2000, 100, "t")])
+def test_dp_bit_exact_with_full_tables(B, k, kind, anchor_stride):
     rng = np.random.default_rng(B * 7 + k)
     if kind == "t":
         h = _t_hist(B, 4096 * 256, seed=k)
@@ -125,6 +136,28 @@ def test_dp_rejects_moment_overflow_on_device():
     with pytest.raises(G.GefenError):
         G.gefen_refit_status(ws)
     assert torch.all(cbo == 7.0)  # outputs untouched
+
+
+def test_dp_full_size_anchored_equals_unanchored():
+    """65536 cells, 256 levels: the anchored search (the automatic choice at
+    this size) and the search of every position over its whole range give the
+    same D and argmin tables bit for bit."""
+    B, k = 65536, 256
+    x = synth.refit_values(4096 * 1024, seed=5, device="cuda")
+    out = []
+    for stride in (-1, 0):
+        G.gefen_refit_debug(stride, 0, 0)
+        try:
+            cbo = torch.empty(k, dtype=torch.float32, device="cuda")
+            ws = G.gefen_refit_codebook(bins=B, k=k, codebook_out=cbo, x=x)
+            G.gefen_refit_status(ws)
+            D, A = G.gefen_refit_tables(ws, B, k)
+            out.append((D.cpu().numpy(), A.cpu().numpy(), cbo.cpu().numpy()))
+        finally:
+            G.gefen_refit_debug(-1, 0, 0)
+    np.testing.assert_array_equal(out[0][0], out[1][0])
+    np.testing.assert_array_equal(out[0][1], out[1][1])
+    np.testing.assert_array_equal(out[0][2], out[1][2])
 
 
 def test_dp_full_size_sampled_entries_and_properties():

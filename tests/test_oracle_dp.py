@@ -245,3 +245,49 @@ def test_dp_entries_reproduce_table_rows():
         np.testing.assert_array_equal(arg, A[lev, lev:])
     val, arg = oracle.dp_entries(h, k, D[k - 1], np.array([b]), last=True)
     assert val[0] == D[k, b] == r["cost"]
+
+
+def _exact_interior(cs, us):
+    s0 = sum(cs)
+    s1 = sum(c * x for c, x in zip(cs, us))
+    s2 = sum(c * x * x for c, x in zip(cs, us))
+    return Fraction(s0 * s2 - s1 * s1, s0)
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_interior_cost_satisfies_the_quadrangle_inequality(seed):
+    """Appendix D's interior cost (squared error of a run of cells about its
+    weighted mean), in exact rationals: for a <= b <= c <= d,
+    cost(a..c) + cost(b..d) <= cost(a..d) + cost(b..c).  The CUDA DP's
+    anchored bracketing rests on this inequality; it also makes the exact
+    smallest minimiser of each DP row non-decreasing in r, checked here on
+    exact rational D rows."""
+    rng = np.random.default_rng(100 + seed)
+    B = 4096
+    h = _rand_hist(rng, B, 40, total=10**7)
+    nz = np.flatnonzero(h)
+    cs = [int(h[i]) for i in nz]
+    us = [2 * int(i) + 1 - B for i in nz]
+    b = len(cs)
+    w = {}
+
+    def cost(l, r):  # 1-based ranks, l <= r
+        if (l, r) not in w:
+            w[(l, r)] = _exact_interior(cs[l - 1:r], us[l - 1:r])
+        return w[(l, r)]
+
+    for _ in range(400):
+        a, bb, c, d = sorted(rng.integers(1, b + 1, 4))
+        assert cost(a, c) + cost(bb, d) <= cost(a, d) + cost(bb, c)
+    # exact D rows for levels 2..4 (first level at -1) and their smallest minimisers
+    first = [None] + [sum(Fraction(cs[j]) * Fraction(us[j] + B) ** 2 for j in range(r)) for r in range(1, b + 1)]
+    prev = first
+    for kk in range(2, 5):
+        row, arg = [None] * (b + 1), [0] * (b + 1)
+        for r in range(kk, b + 1):
+            vals = [(prev[l - 1] + cost(l, r), l) for l in range(kk, r + 1)]
+            best = min(v for v, _ in vals)
+            row[r] = best
+            arg[r] = min(l for v, l in vals if v == best)
+        assert all(arg[r] <= arg[r + 1] for r in range(kk, b))
+        prev = row

@@ -58,6 +58,43 @@ def test_static_refit_matches_workspace_refit_on_two_calls_in_a_row():
     assert got1["cb"][0] == -1.0 and got1["cb"][-1] == 1.0
 
 
+def test_static_refit_allocates_nothing():
+    # init first (module, array and kernels loaded), then no call changes the
+    # device's free memory, outputs being allocated beforehand
+    G.gefen_refit_static_init()
+    x = synth.refit_values(4096 * 256, seed=13, device="cuda")
+    cb = torch.empty(256, dtype=torch.float32, device="cuda")
+    ho = torch.zeros(4096, dtype=torch.int64, device="cuda")
+    G.gefen_refit_codebook_static(bins=4096, k=256, codebook_out=cb, x=x, hist_out=ho)
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    for _ in range(2):
+        ho.zero_()
+        G.gefen_refit_codebook_static(bins=4096, k=256, codebook_out=cb, x=x, hist_out=ho)
+    assert G.gefen_refit_static_status() == 256
+    torch.cuda.synchronize()
+    assert torch.cuda.mem_get_info()[0] == free0
+
+
+def test_static_refit_reports_moment_overflow():
+    # N (B-1)^2 >= 2^64: the device-side check fails, the outputs stay as
+    # they were and the static status call reports it
+    B, k = 4096, 4
+    h = np.zeros(B, np.int64)
+    h[[0, 7, B - 1]] = 1 << 40
+    hd = torch.from_numpy(h).cuda()
+    cb = torch.full((k,), 7.0, device="cuda")
+    G.gefen_refit_codebook_static(bins=B, k=k, codebook_out=cb, hist_in=hd)
+    with pytest.raises(G.GefenError) as e:
+        G.gefen_refit_static_status()
+    assert e.value.status == G.GEFEN_EDEVICE
+    assert torch.all(cb == 7.0)
+    # and a valid histogram afterwards is refit normally
+    h2 = torch.from_numpy(np.arange(1, B + 1, dtype=np.int64)).cuda()
+    G.gefen_refit_codebook_static(bins=B, k=k, codebook_out=cb, hist_in=h2)
+    assert G.gefen_refit_static_status() == k
+
+
 def test_static_refit_rejects_sizes_beyond_its_array():
     cb = torch.empty(256, dtype=torch.float32, device="cuda")
     h = torch.ones(8192, dtype=torch.int64, device="cuda")
