@@ -497,6 +497,7 @@ int64_t oracle_infer_blocks(const uint16_t* grad, int64_t n, double eps,
     double* S = (double*)malloc(sizeof(double) * (size_t)nd);
     double* z = (double*)malloc(sizeof(double) * (size_t)n);
     oracle_divisors(n, P, nd);
+    #pragma omp parallel for schedule(static)
     for (int64_t j = 0; j < n; ++j) {
         double g = bf16_to_double(grad[j]);
         z[j] = log(g * g + eps);

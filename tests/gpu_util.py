@@ -172,3 +172,26 @@ def ambiguous_bins(x64, bins):
         t = (x.astype(np.float32) + np.float32(1.0)).astype(np.float32) * np.float32(0.5 * bins)
         return np.clip(np.floor(t), 0, bins - 1)
     return int(np.count_nonzero(cell(x64 * (1 - MARGIN)) != cell(x64 * (1 + MARGIN))))
+
+
+_ORACLE_PERIODS = {}
+
+
+def oracle_model_periods(name: str, seed: int, grads_host=None):
+    """The oracle's periods (Algorithm 2) for every tensor of a model-shaped
+    set, from its first gradient as the bench draws it (seed, step 1); cached
+    per (set, seed) for the test session.  Returns (periods, scores)."""
+    from paper_2606_13894_gb300 import synth
+    key = (name, seed)
+    if key not in _ORACLE_PERIODS:
+        specs = synth.CONFIGS[name]()
+        offs, _ = synth.pack_offsets(specs)
+        if grads_host is None:
+            grads_host = bits(synth.draw_grads(specs, seed, step=1, device="cuda"))
+        periods, scores = [], []
+        for s, o in zip(specs, offs):
+            p, _, sc = oracle.infer_blocks(grads_host[o:o + s.numel])
+            periods.append(p)
+            scores.append(sc)
+        _ORACLE_PERIODS[key] = (periods, scores)
+    return _ORACLE_PERIODS[key]
