@@ -12,12 +12,19 @@ learned from it.
 `--workload flat:N:P` runs one flat tensor of N parameters with blocks of P
 (given, not inferred): the small case the kernel profiles are taken on.
 
+Under torchrun with N ranks the model is block-sharded over the ranks
+(paper_2606_13894_gb300/shard.py): each rank steps its own blocks, and a refit
+sums the ranks' histograms with one all-reduce before every rank runs the same
+DP.  The model is fixed, so N ranks scale it strongly.
+
 Prints one JSON line.  `value` is whole-job parameters updated per second over
 the timed steps (refit steps included); `e2e` is the same metric through the
 public call with the gradient copied in from pinned host memory and the step's
 status word read back every step (and, as a second figure, all updated
-parameters copied back too).  `--impl reference` times the CPU oracle instead, on a bounded
-sample of the same workload.
+parameters copied back too).  On one GPU the line also carries the same job
+with 65536-cell refits, the GPT-2-125M-shaped set and a flat sweep.
+`--impl reference` times the CPU oracle instead, on a bounded sample of the
+same workload.
 """
 from __future__ import annotations
 
@@ -150,10 +157,11 @@ def job_time_ms(elapsed_ms: float, world: int, device) -> float:
     return float(t.item())
 
 
-def whole_job_value(params_per_rank: int, world: int, steps: int, job_ms: float) -> float:
-    """Parameters all replicas updated per second (each rank steps its own
-    copy of the workload: weak scaling), in Gparams/s."""
-    return world * params_per_rank * steps / (job_ms * 1e-3) / 1e9
+def whole_job_value(params_total: int, steps: int, job_ms: float) -> float:
+    """Parameters of the model updated per second, in Gparams/s: the ranks
+    share one model (each steps its own blocks), so this is the model's
+    parameter count over the slowest rank's time per step."""
+    return params_total * steps / (job_ms * 1e-3) / 1e9
 
 
 def dist_env():
@@ -209,6 +217,121 @@ def period_summary(specs, periods):
 
 
 # ----------------------------------------------------------------- GPU arm
+def infer_periods(G, specs, grads, dev):
+    """Algorithm 2 on the first gradient of every tensor (arena `grads`)."""
+    from paper_2606_13894_gb300 import synth
+    offs, _ = synth.pack_offsets(specs)
+    periods, iws = [], None
+    for s, o in zip(specs, offs):
+        need = G.gefen_infer_workspace_size(s.numel)
+        if iws is None or iws.numel() < need:
+            iws = G.workspace(need, dev)
+        p, _ = G.gefen_infer_blocks(grads[o:o + s.numel], HP["eps"], workspace_buf=iws, want_scores=False)
+        periods.append(p)
+    return periods
+
+
+def make_shard(G, synth, dev, specs, periods, rank, world, group, bins, refit_every, split):
+    """This rank's shard of the workload (block-aligned; the whole model on
+    one rank) with its parameters and a pool of two gradients (steps 1, 2)."""
+    from paper_2606_13894_gb300 import shard
+    sh = shard.RankShard([(s.numel, p) for s, p in zip(specs, periods)], rank, world, dev, levels=K, bins=bins,
+                         refit_every=refit_every, group=group, split=split)
+    offs, _ = synth.pack_offsets(specs)
+    if world == 1:  # the rank's arena is the model's arena
+        synth.init_params(specs, SEED, device=dev, out=sh.theta)
+        gpool = [synth.draw_grads(specs, SEED, step=s, device=dev) for s in (1, 2)]
+    else:
+        th = synth.init_params(specs, SEED, device=dev)
+        sh.gather(lambda i: th[offs[i]:offs[i] + specs[i].numel], torch.float32, out=sh.theta)
+        del th
+        gpool = []
+        for s in (1, 2):
+            g = synth.draw_grads(specs, SEED, step=s, device=dev)
+            gpool.append(sh.gather(lambda i: g[offs[i]:offs[i] + specs[i].numel], torch.bfloat16))
+            del g
+    torch.cuda.synchronize()
+    return sh, gpool
+
+
+class Cadence:
+    """The workload's steps on one rank's shard (refit every REFIT_EVERY
+    steps), with CUDA events on the launching stream: plain steps, the first
+    call of a plain step (the dominant kernel's tensors, when the step is
+    split), refit steps (step, then DP)."""
+
+    def __init__(self, sh, gpool, stream, hp, dominant_first: bool):
+        self.sh, self.gpool, self.stream, self.hp = sh, gpool, stream, hp
+        self.dominant_first = dominant_first
+        self.plain, self.dom, self.refit = [], [], []
+
+    def _ev(self):
+        e = torch.cuda.Event(enable_timing=True)
+        e.record(self.stream)
+        return e
+
+    def step(self, timed: bool, g=None) -> bool:
+        sh = self.sh
+        if g is None:
+            g = self.gpool[(sh.t + 1) % 2]
+        e0 = self._ev() if timed else None
+        ea = []
+
+        def after(i):
+            if timed and i == 0 and self.dominant_first:
+                ea.append(self._ev())
+
+        refit = sh.step_local(g, self.hp, after_call=after)
+        e1 = self._ev() if timed else None
+        if refit:
+            sh.refit_codebook()
+            if timed:
+                self.refit.append((e0, e1, self._ev()))
+        elif timed:
+            self.plain.append((e0, e1))
+            if ea:
+                self.dom.append((e0, ea[0]))
+        return refit
+
+    def reset_events(self):
+        self.plain, self.dom, self.refit = [], [], []
+
+    def mean_ms(self, which: str, part: int = 0):
+        ev = getattr(self, which)
+        if not ev:
+            return None
+        if which == "refit":
+            return statistics.mean(e[part].elapsed_time(e[part + 1]) for e in ev)
+        return statistics.mean(a.elapsed_time(b) for a, b in ev)
+
+
+def timed_steps(cad: Cadence, steps: int, warm: int, stream, world: int, dev, clocks=None):
+    """warm untimed steps, then `steps` timed ones bracketed by a barrier and
+    synchronisation; returns the job time (slowest rank) in ms."""
+    for _ in range(warm):
+        cad.step(False)
+    torch.cuda.synchronize()
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    torch.cuda.synchronize()
+    cad.reset_events()
+    if clocks is not None:
+        clocks.start()
+        time.sleep(0.15)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(steps):
+        cad.step(True)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    ck = None
+    if clocks is not None:
+        time.sleep(0.05)
+        ck = clocks.stop()
+    return job_time_ms(ev0.elapsed_time(ev1), world, dev), ck
+
+
 def run_gpu(args, world, rank, local):
     from paper_2606_13894_gb300 import gefen as G
     from paper_2606_13894_gb300 import synth
@@ -216,188 +339,179 @@ def run_gpu(args, world, rank, local):
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     G.load()
-    specs, given_periods = workload_specs(synth, args.workload)
-    offs, total = synth.pack_offsets(specs)
-    nparams = synth.total_params(specs)
-    stream = torch.cuda.current_stream()
-
-    theta = synth.init_params(specs, SEED + rank, device=dev)
-    gpool = [synth.draw_grads(specs, SEED + rank, step=s, device=dev) for s in (1, 2)]
-    torch.cuda.synchronize()
-
-    # Algorithm 2 on the first gradient of every tensor
-    t0 = time.perf_counter()
-    periods = list(given_periods) if given_periods else []
-    iws = None
-    for s, o in zip(specs, offs) if not given_periods else []:
-        need = G.gefen_infer_workspace_size(s.numel)
-        if iws is None or iws.numel() < need:
-            iws = G.workspace(need, dev)
-        p, _ = G.gefen_infer_blocks(gpool[0][o:o + s.numel], HP["eps"], workspace_buf=iws, want_scores=False)
-        periods.append(p)
-    infer_s = time.perf_counter() - t0
-    del iws
-    entries, boff = [], 0
-    for s, o, p in zip(specs, offs, periods):
-        entries.append((o, s.numel, p, boff))
-        boff += s.numel // p
-    nblocks = boff
-    table = G.tensor_table(entries)
-    # a step is two calls: the tensors of the dominant kernel, then the rest,
-    # so CUDA events time that kernel's launch on its own
-    ent_a = [e for e in entries if dominant(e[2])]
-    ent_b = [e for e in entries if not dominant(e[2])]
-    table_a, table_b = G.tensor_table(ent_a), G.tensor_table(ent_b)
-    n_a = sum(e[1] for e in ent_a)
-    blocks_a = sum(e[1] // e[2] for e in ent_a)
-    codes = torch.empty(total, dtype=torch.uint8, device=dev)
-    v = torch.zeros(nblocks, dtype=torch.float32, device=dev)
-    sc = torch.zeros(nblocks, dtype=torch.float32, device=dev)
-    hist = torch.zeros(BINS, dtype=torch.int64, device=dev)
-    cb = torch.empty(K, dtype=torch.float32, device=dev)
-    cb_new = torch.empty(K, dtype=torch.float32, device=dev)
-
-    # Algorithm 3 on the first gradient: histogram of g / block absmax, DP
-    ws = G.workspace(G.gefen_step_workspace_size(table, G.GEFEN_HIST), dev)
-    ws_b = G.workspace(G.gefen_step_workspace_size(table_b, G.GEFEN_HIST), dev)
-    rws = G.workspace(G.gefen_refit_workspace_size(BINS, K), dev)
-    t0 = time.perf_counter()
-    G.gefen_step(table, theta, gpool[0], codes, v, sc, cb, cb, step=1, flags=G.GEFEN_HIST_GRAD_ONLY,
-                 hist=hist, workspace_buf=ws, **HP)
-    G.gefen_refit_codebook(bins=BINS, k=K, codebook_out=cb, hist_in=hist, workspace_buf=rws)
-    G.gefen_refit_status(rws)
-    init_codebook_s = time.perf_counter() - t0
-    zc = int(torch.argmin(cb.abs()).item())
-    codes.fill_(zc)
-
-    step_events = []   # (start, end) of plain steps
-    dom_events = []    # (start, end) of the dominant kernel's call in plain steps
-    refit_events = []  # (step start, step end, dp end)
-    state = {"t": 0, "switch": False}
-
-    def one_step(timed: bool):
-        state["t"] += 1
-        t = state["t"]
-        g = gpool[t % 2]
-        refit = (t % REFIT_EVERY == 0)
-        enc = cb_new if state["switch"] else cb
-        e0 = torch.cuda.Event(enable_timing=True) if timed else None
-        e1 = torch.cuda.Event(enable_timing=True) if timed else None
-        e2 = torch.cuda.Event(enable_timing=True) if timed and refit else None
-        ea = torch.cuda.Event(enable_timing=True) if timed and not refit else None
-        if timed:
-            e0.record(stream)
-        flags = G.GEFEN_HIST if refit else 0
-        if refit:
-            hist.zero_()
-        G.gefen_step(table_a, theta, g, codes, v, sc, cb, enc, step=t, flags=flags, hist=hist if refit else None,
-                     workspace_buf=ws, **HP)
-        if ea is not None:
-            ea.record(stream)
-            dom_events.append((e0, ea))
-        G.gefen_step(table_b, theta, g, codes, v, sc, cb, enc, step=t, flags=flags, hist=hist if refit else None,
-                     workspace_buf=ws_b, **HP)
-        if timed:
-            e1.record(stream)
-        if state["switch"]:
-            cb.copy_(cb_new)
-            state["switch"] = False
-        if refit:
-            G.gefen_refit_codebook(bins=BINS, k=K, codebook_out=cb_new, hist_in=hist, workspace_buf=rws)
-            state["switch"] = True
-            if timed:
-                e2.record(stream)
-                refit_events.append((e0, e1, e2))
-        elif timed:
-            step_events.append((e0, e1))
-
-    warm = max(3, args.warmup)
-    for _ in range(warm):
-        one_step(False)
-    torch.cuda.synchronize()
-
     group = None
     if world > 1:
         import torch.distributed as dist
         group = dist.group.WORLD
-        dist.barrier()
-    torch.cuda.synchronize()
-    clocks = Clocks(local)
-    clocks.start()
-    time.sleep(0.15)
-    ev0 = torch.cuda.Event(enable_timing=True)
-    ev1 = torch.cuda.Event(enable_timing=True)
-    ev0.record(stream)
-    for _ in range(args.steps):
-        one_step(True)
-    ev1.record(stream)
-    torch.cuda.synchronize()
-    time.sleep(0.05)
-    ck = clocks.stop()
-    G.gefen_step_status(ws)  # raises if a bounded device wait gave up
-    G.gefen_step_status(ws_b)
-    elapsed_ms = job_time_ms(ev0.elapsed_time(ev1), world, dev)
+    specs, given_periods = workload_specs(synth, args.workload)
+    nparams = synth.total_params(specs)
+    stream = torch.cuda.current_stream()
 
-    plain_ms = [a.elapsed_time(b) for a, b in step_events]
-    refit_step_ms = [a.elapsed_time(b) for a, b, _ in refit_events]
-    dp_ms = [b.elapsed_time(c) for _, b, c in refit_events]
-    avg_step_ms = statistics.mean(plain_ms) if plain_ms else float("nan")
+    # Algorithm 2 on the first gradient of every tensor: every rank infers
+    # the same blocks from the same gradient
+    t0 = time.perf_counter()
+    if given_periods:
+        periods = given_periods * len(specs)
+    else:
+        g1 = synth.draw_grads(specs, SEED, step=1, device=dev)
+        periods = infer_periods(G, specs, g1, dev)
+        del g1
+    infer_s = time.perf_counter() - t0
+    # a step is two calls on each rank: the tensors of the dominant kernel,
+    # then the rest, so CUDA events time that kernel's launch on its own
+    sh, gpool = make_shard(G, synth, dev, specs, periods, rank, world, group, BINS, REFIT_EVERY, dominant)
+    dom_first = bool(sh.call_entries) and all(dominant(e[2]) for e in sh.call_entries[0])
+    n_rank, blocks_rank = sh.numel, sum(pc.nblocks for pc in sh.pieces)
+    n_a = sum(e[1] for e in sh.call_entries[0]) if dom_first else 0
+    blocks_a = sum(e[1] // e[2] for e in sh.call_entries[0]) if dom_first else 0
+    nblocks = sum(s.numel // p for s, p in zip(specs, periods))
 
-    alg_bytes = 12 * nparams + 16 * nblocks + 8 * K
+    # Algorithm 3 on the first gradient: histogram of g / block absmax (summed
+    # over the ranks), then the exact DP
+    t0 = time.perf_counter()
+    sh.init_codebook(gpool[0], HP)
+    G.gefen_refit_status(sh.rws)
+    init_codebook_s = time.perf_counter() - t0
+
+    cad = Cadence(sh, gpool, stream, HP, dom_first)
+    warm = max(3, args.warmup)
+    elapsed_ms, ck = timed_steps(cad, args.steps, warm, stream, world, dev, clocks=Clocks(local))
+    G.gefen_step_status(sh.ws)  # raises if a bounded device wait gave up
+    G.gefen_refit_status(sh.rws)
+
+    avg_step_ms = cad.mean_ms("plain")
+    dom_ms = cad.mean_ms("dom")
     hbm, peak_kind = peaks()
-    # the dominant kernel alone: 12 bytes per parameter and 16 per block
-    dom_ms = statistics.mean([a.elapsed_time(b) for a, b in dom_events]) if dom_events else float("nan")
+    alg_bytes = 12 * n_rank + 16 * blocks_rank + 8 * K
     alg_bytes_a = 12 * n_a + 16 * blocks_a
-    achieved = alg_bytes_a / (dom_ms * 1e-3) / 1e9
-    traffic = profiled_traffic(n_a)
+    achieved = alg_bytes_a / (dom_ms * 1e-3) / 1e9 if dom_ms else None
+    traffic = profiled_traffic(n_a) if dom_first else None
 
-    # e2e: gradient in from pinned host memory, parameters back, every step
-    e2e = None
-    if rank == 0 or world > 1:
-        e2e = run_e2e(G, table, theta, codes, v, sc, cb, ws, gpool, nparams, stream, args, state, one_step_ctx=(
-            hist, cb_new, rws))
+    e2e = run_e2e(G, cad, args, stream)
 
-    per_a = [e[2] for e in ent_a]
-    per_b = [e[2] for e in ent_b]
-    n_launch_plain = launches_per_call(per_a, False) + launches_per_call(per_b, False)
-    # refit steps: one histogram per call, then the DP: prefix, levels 1..K-1 and the last, backtrack
-    n_launch_refit = launches_per_call(per_a, True) + launches_per_call(per_b, True) + 1 + (K - 1) + 1
-    nref = len(refit_events)
+    per = [[e[2] for e in ce] for ce in sh.call_entries]
+    n_launch_plain = sum(launches_per_call(x, False) for x in per)
+    # refit steps: the step's calls with their histograms, then the DP's four
+    # launches (prefix, first level, the cooperative levels launch, backtrack)
+    n_launch_refit = sum(launches_per_call(x, True) for x in per) + 4
+    nref = len(cad.refit)
     launches = (args.steps - nref) * n_launch_plain + nref * n_launch_refit
 
+    whole_step_ms = avg_step_ms
     res = {
-        "metric": METRIC, "value": whole_job_value(nparams, world, args.steps, elapsed_ms), "unit": UNIT,
+        "metric": METRIC, "value": whole_job_value(nparams, args.steps, elapsed_ms), "unit": UNIT,
         "n_gpus": world, "steps": args.steps, "warmup": warm, "ms_per_step": elapsed_ms / args.steps,
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "higher_is_better": True, "scaling": "strong", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic (seeded; shapes and gradient-scale structure of the Llama-3-1.5B run)",
         "config": {"workload": f"{args.workload} shaped set: {len(specs)} tensors, {nparams} fp32 params, "
                                f"{nblocks} inferred blocks; 256-level codebook; refit every {REFIT_EVERY} "
-                               f"steps with {BINS} cells",
+                               f"steps with {BINS} cells (16 per level: Algorithm 3's 16k cells read as 16 k); "
+                               f"the same job with 65536-cell refits is under refit_65536",
                    "params": nparams, "tensors": len(specs), "blocks": nblocks, "refit_every": REFIT_EVERY,
                    "bins": BINS, "levels": K, "hparams": HP,
                    "l2": "inputs larger than L2: 17.7 GB of step traffic per step, no flush needed",
-                   "parallelism": "replicas" if world > 1 else "single GPU"},
+                   "parallelism": ("single GPU" if world == 1 else
+                                   f"block-sharded over {world} ranks ({n_rank} params on rank {rank}); "
+                                   f"one histogram all-reduce per refit")},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                     "frac": achieved / hbm, "traffic": traffic,
+                     "frac": achieved / hbm if achieved else None, "traffic": traffic,
                      "kernel": DOMINANT, "peak_kind": peak_kind,
                      "alg_bytes_per_launch": alg_bytes_a, "params_per_launch": n_a, "blocks_per_launch": blocks_a,
                      "avg_launch_ms": dom_ms,
-                     "whole_step": {"alg_bytes": alg_bytes, "avg_ms": avg_step_ms,
-                                    "achieved_gbs": alg_bytes / (avg_step_ms * 1e-3) / 1e9}},
-        "step_only": {"value": nparams / (avg_step_ms * 1e-3) / 1e9 if plain_ms else None, "unit": UNIT,
-                      "ms": avg_step_ms},
-        "refit": {"dp_ms": statistics.mean(dp_ms) if dp_ms else None,
-                  "hist_step_ms": statistics.mean(refit_step_ms) if refit_step_ms else None,
-                  "count": nref},
+                     "whole_step": {"alg_bytes": alg_bytes, "avg_ms": whole_step_ms,
+                                    "achieved_gbs": alg_bytes / (whole_step_ms * 1e-3) / 1e9,
+                                    "frac": alg_bytes / (whole_step_ms * 1e-3) / 1e9 / hbm}},
+        "step_only": {"value": nparams / (avg_step_ms * 1e-3) / 1e9 if avg_step_ms else None,
+                      "unit": UNIT, "ms": avg_step_ms},
+        "refit": {"dp_ms": cad.mean_ms("refit", 1), "hist_step_ms": cad.mean_ms("refit", 0), "count": nref},
         "init": {"infer_blocks_s": infer_s, "first_codebook_s": init_codebook_s},
         "periods": period_summary(specs, periods),
         "e2e": e2e, "gpu_launches": launches, "clocks": ck,
     }
+    if world == 1 and not args.no_extras:
+        res["refit_65536"] = cadence_65536(G, cad, args, stream, dev, nparams)
+    del cad, sh, gpool
+    torch.cuda.empty_cache()
     if rank == 0 and not args.no_microbench:
         res["refit_microbench"] = refit_microbench(G, synth, dev, args.micro_values, args.micro_bins)
+    if world == 1 and not args.no_extras:
+        res["gpt2_125m"] = gpt2_figures(G, synth, dev, args, stream, hbm)
+        res["flat_sweep"] = flat_sweep(G, synth, dev, stream, hbm)
     if rank == 0 and not args.no_cpu_baseline:
         res["cpu_baseline"] = cpu_baseline(args)
     return res
+
+
+def cadence_65536(G, cad, args, stream, dev, nparams):
+    """The same job with refits from 65536-cell histograms (SURVEY's reading
+    for this set): the x of every tensor is staged and counted by the
+    65536-cell histogram kernel, then the 65536 x 256 DP."""
+    sh = cad.sh
+    sh.set_refit_bins(65536)
+    cad.reset_events()
+    ms, _ = timed_steps(cad, args.steps, 3, stream, 1, dev)
+    G.gefen_refit_status(sh.rws)
+    out = {"value": whole_job_value(nparams, args.steps, ms), "unit": UNIT, "ms_per_step": ms / args.steps,
+           "steps": args.steps, "refit_every": REFIT_EVERY, "bins": 65536,
+           "dp_ms": cad.mean_ms("refit", 1), "hist_step_ms": cad.mean_ms("refit", 0), "count": len(cad.refit)}
+    sh.set_refit_bins(BINS)
+    return out
+
+
+GPT2_HP = dict(lr=6e-4, beta1=0.9, beta2=0.95, eps=1e-8, weight_decay=0.1)  # Appendix I, GPT-2
+
+
+def gpt2_figures(G, synth, dev, args, stream, hbm):
+    """The GPT-2-125M-shaped set (blocks inferred from its first gradient):
+    the whole job with the same refit cadence, and a plain step's throughput
+    and algorithmic bytes per second."""
+    specs = synth.gpt2_125m_set()
+    n = synth.total_params(specs)
+    g1 = synth.draw_grads(specs, SEED, step=1, device=dev)
+    periods = infer_periods(G, specs, g1, dev)
+    del g1
+    sh, gpool = make_shard(G, synth, dev, specs, periods, 0, 1, None, BINS, REFIT_EVERY, None)
+    sh.init_codebook(gpool[0], GPT2_HP)
+    cad = Cadence(sh, gpool, stream, GPT2_HP, False)
+    steps = max(args.steps, 20)
+    ms, _ = timed_steps(cad, steps, 3, stream, 1, dev)
+    G.gefen_step_status(sh.ws)
+    step_ms = cad.mean_ms("plain")
+    nb = sum(s.numel // p for s, p in zip(specs, periods))
+    alg = 12 * n + 16 * nb + 8 * K
+    out = {"params": n, "blocks": nb, "hparams": GPT2_HP,
+           "whole_job": {"value": whole_job_value(n, steps, ms), "unit": UNIT, "ms_per_step": ms / steps,
+                         "steps": steps, "refit_every": REFIT_EVERY, "bins": BINS},
+           "step": {"value": n / (step_ms * 1e-3) / 1e9, "unit": UNIT, "ms": step_ms,
+                    "alg_bytes": alg, "achieved_gbs": alg / (step_ms * 1e-3) / 1e9,
+                    "frac": alg / (step_ms * 1e-3) / 1e9 / hbm},
+           "periods": period_summary(specs, periods),
+           "l2": "1.5 GB of step traffic per step against a 129 MB L2: no flush needed"}
+    del cad, sh, gpool
+    torch.cuda.empty_cache()
+    return out
+
+
+def flat_sweep(G, synth, dev, stream, hbm, sizes=(1 << 28, 1 << 31)):
+    """One flat tensor of N fp32 parameters with given blocks of p: a plain
+    step's time and algorithmic GB/s (12 B per parameter and 16 per block)."""
+    out = {}
+    for n in sizes:
+        for p in (1, 64, 4096, 1 << 20, n):
+            specs = synth.flat_set(n, p)
+            sh, gpool = make_shard(G, synth, dev, specs, [p], 0, 1, None, BINS, 0, None)
+            sh.init_codebook(gpool[0], HP)
+            cad = Cadence(sh, gpool, stream, HP, False)
+            timed_steps(cad, 5, 3, stream, 1, dev)
+            G.gefen_step_status(sh.ws)
+            ms = cad.mean_ms("plain")
+            alg = 12 * n + 16 * (n // p)
+            out[f"2^{n.bit_length() - 1}/{'n' if p == n else p}"] = {
+                "ms": ms, "gparams": n / (ms * 1e-3) / 1e9, "achieved_gbs": alg / (ms * 1e-3) / 1e9,
+                "frac": alg / (ms * 1e-3) / 1e9 / hbm}
+            del cad, sh, gpool
+            torch.cuda.empty_cache()
+    return out
 
 
 def refit_microbench(G, synth, dev, n=MICRO_N, bins=MICRO_BINS):
@@ -427,31 +541,28 @@ def refit_microbench(G, synth, dev, n=MICRO_N, bins=MICRO_BINS):
             "hist_gbs": 4 * n / ((hist_dp_ms - dp_ms) * 1e-3) / 1e9}
 
 
-def run_e2e(G, table, theta, codes, v, sc, cb, ws, gpool, nparams, stream, args, state, one_step_ctx):
-    """Same step through the public API with host buffers: every step copies
-    its bf16 gradient in from pinned memory, runs gefen_step and reads the
-    step's result back (its 4-byte status word, gefen_step_status, which
-    waits for the step).  A second figure also copies all updated fp32
-    parameters back to pinned memory every step."""
-    hist, cb_new, rws = one_step_ctx
-    n = gpool[0].numel()
+def run_e2e(G, cad, args, stream):
+    """The same job through the public API with host buffers: every step
+    copies its bf16 gradient in from pinned memory and runs the step (refit
+    steps included, with the timed region's cadence and step count), and the
+    step's result is read back: its 4-byte status word (gefen_step_status,
+    which waits for the step).  A second figure also copies the rank's
+    updated fp32 parameters back to pinned memory every step."""
+    sh = cad.sh
+    n = sh.numel_arena
     g_host = torch.empty(n, dtype=torch.bfloat16, pin_memory=True)
-    th_host = torch.empty(theta.numel(), dtype=torch.float32, pin_memory=True)
-    g_host.copy_(gpool[1])
-    gdev = torch.empty_like(gpool[0])
-    steps = max(3, min(args.steps, 10))
+    th_host = torch.empty(n, dtype=torch.float32, pin_memory=True)
+    g_host.copy_(cad.gpool[1])
+    gdev = torch.empty_like(cad.gpool[0])
+    steps = args.steps
 
     def e2e_step(readback_params: bool):
-        state["t"] += 1
         gdev.copy_(g_host, non_blocking=True)
-        G.gefen_step(table, theta, gdev, codes, v, sc, cb, cb, step=state["t"], workspace_buf=ws, **HP)
+        cad.step(False, g=gdev)
         if readback_params:
-            th_host.copy_(theta, non_blocking=True)
-        G.gefen_step_status(ws)
+            th_host.copy_(sh.theta, non_blocking=True)
+        G.gefen_step_status(sh.ws)
 
-    if state["switch"]:
-        cb.copy_(cb_new)
-        state["switch"] = False
     out = {}
     for key, rb in (("status", False), ("params", True)):
         for _ in range(2):
@@ -462,11 +573,13 @@ def run_e2e(G, table, theta, codes, v, sc, cb, ws, gpool, nparams, stream, args,
             e2e_step(rb)
         torch.cuda.synchronize()
         out[key] = time.perf_counter() - t0
+    nparams = sum(pc.numel for pc in sh.pieces)
     return {"value": nparams * steps / out["status"] / 1e9, "unit": UNIT, "steps": steps,
+            "refit_every": sh.refit_every,
             "h2d_bytes_per_step": 2 * n, "d2h_bytes_per_step": 4,
             "result_read": "the step's status word (gefen_step_status), every step",
             "with_params_readback": {"value": nparams * steps / out["params"] / 1e9, "unit": UNIT,
-                                     "h2d_bytes_per_step": 2 * n, "d2h_bytes_per_step": 4 * theta.numel() + 4}}
+                                     "h2d_bytes_per_step": 2 * n, "d2h_bytes_per_step": 4 * n + 4}}
 
 
 # ------------------------------------------------------------ CPU oracle arm
@@ -510,23 +623,53 @@ def oracle_steps(data, cb, t):
     return time.perf_counter() - t0
 
 
+def host_cpu():
+    """Host CPU model name (lscpu) and logical core count."""
+    name = None
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.lower().startswith("model name"):
+                name = line.split(":", 1)[1].strip()
+                break
+    except Exception:
+        pass
+    return {"model": name, "nproc": os.cpu_count()}
+
+
 def cpu_baseline(args):
+    """The oracle's step on the host: single-threaded and with its loop over
+    blocks on every core (the figure reported as `value`)."""
     import oracle
     data, cb, done = oracle_sample_data(args.cpu_params, args.workload)
-    secs, t = 0.0, 0
-    while secs < args.cpu_budget or t == 0:
-        t += 1
-        secs += oracle_steps(data, cb, t)
-    return {"value": done * t / secs / 1e9, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"{t} oracle steps (single thread, double precision) over {len(data)} whole tensors "
-                      f"of the {args.workload} set ({done} params: {data[0]['name']} .. {data[-1]['name']}), "
-                      f"{secs:.1f} s",
-            "threads_available": os.cpu_count(), "oracle_threads": oracle.num_threads()}
+    runs = {}
+    ncores = os.cpu_count() or 1
+    t = 0
+    for threads in (1, ncores):
+        oracle.set_num_threads(threads)
+        secs, steps = 0.0, 0
+        while secs < args.cpu_budget / 2 or steps == 0:
+            t += 1
+            steps += 1
+            secs += oracle_steps(data, cb, t)
+        runs[threads] = (done * steps / secs / 1e9, steps, secs)
+    oracle.set_num_threads(ncores)
+    val, steps, secs = runs[ncores]
+    return {"value": val, "unit": UNIT, "cores": ncores, "kind": "oracle",
+            "sample": f"{steps} oracle steps (double precision, its loop over blocks on {ncores} threads) over "
+                      f"{len(data)} whole tensors of the {args.workload} set ({done} params: {data[0]['name']} .. "
+                      f"{data[-1]['name']}), {secs:.1f} s",
+            "single_thread": {"value": runs[1][0], "unit": UNIT, "cores": 1, "steps": runs[1][1],
+                              "seconds": runs[1][2]},
+            "host": host_cpu()}
 
 
 def run_reference(args, world, rank):
     if rank != 0:
         return None
+    import oracle
+    ncores = os.cpu_count() or 1
+    oracle.set_num_threads(ncores)
     warm = max(3, args.warmup)
     data, cb, done = oracle_sample_data(int(args.ref_params), args.workload)
     t = 0
@@ -544,8 +687,10 @@ def run_reference(args, world, rank):
             "data": "synthetic (seeded)",
             "config": {"workload": f"{args.workload} shaped set, bounded sample: {len(data)} whole tensors "
                                    f"({done} params) per step, oracle step"},
-            "cpu_baseline": {"value": val, "unit": UNIT, "cores": 1, "kind": "oracle",
-                             "sample": f"{done} params per step ({len(data)} tensors of the {args.workload} set)"},
+            "cpu_baseline": {"value": val, "unit": UNIT, "cores": ncores, "kind": "oracle",
+                             "sample": f"{done} params per step ({len(data)} tensors of the {args.workload} set), "
+                                       f"the oracle's loop over blocks on {ncores} threads",
+                             "host": host_cpu()},
             "e2e": {"value": val, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
@@ -560,6 +705,8 @@ def main():
     ap.add_argument("--ref-params", type=float, default=20e6, help="oracle params per reference step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-microbench", action="store_true", help="skip the 65536-cell refit measurement")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="skip the 65536-cell cadence, GPT-2-125M and flat-sweep figures")
     ap.add_argument("--microbench-only", action="store_true",
                     help="run only the refit micro-benchmark and print its figures (one GPU)")
     ap.add_argument("--micro-values", type=int, default=MICRO_N, help="refit micro-benchmark values (multiple of 4096)")

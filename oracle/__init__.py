@@ -57,6 +57,8 @@ def _load():
     P = ctypes.c_void_p
     i64, i32, f64 = ctypes.c_int64, ctypes.c_int32, ctypes.c_double
     lib.oracle_num_threads.restype = ctypes.c_int
+    lib.oracle_set_num_threads.argtypes = [ctypes.c_int32]
+    lib.oracle_set_num_threads.restype = None
     lib.oracle_bin.argtypes = [ctypes.c_float, i32]
     lib.oracle_bin.restype = i64
     lib.oracle_histogram.argtypes = [P, i64, i32, P]
@@ -88,6 +90,11 @@ def _load():
 def _ptr(a: np.ndarray):
     assert a.flags.c_contiguous, "oracle arrays must be C-contiguous"
     return a.ctypes.data_as(ctypes.c_void_p)
+
+
+def set_num_threads(n: int) -> None:
+    """Threads of the oracle's parallel loops (results do not depend on it)."""
+    _load().oracle_set_num_threads(int(n))
 
 
 def num_threads() -> int:

@@ -41,6 +41,16 @@ int oracle_num_threads(void) {
 #endif
 }
 
+/* Threads of the parallel loops below (blocks of a step, divisors, rows of a
+ * DP level); every result is the same for any count. */
+void oracle_set_num_threads(int32_t n) {
+#ifdef _OPENMP
+    if (n > 0) omp_set_num_threads(n);
+#else
+    (void)n;
+#endif
+}
+
 /* bf16 bit pattern -> float (exact: bf16 is the upper half of an fp32). */
 static double bf16_to_double(uint16_t b) {
     uint32_t u = ((uint32_t)b) << 16;
@@ -120,10 +130,16 @@ int oracle_step(int64_t n, int64_t p, float* theta, const uint16_t* grad,
     const double bc1 = 1.0 - pow(beta1, (double)t);
     const double bc2 = 1.0 - pow(beta2, (double)t);
     const int zero_code = nearest_level(0.0, cb_enc, k);
+    int failed = 0;
+    /* blocks are independent (each thread keeps its own m); histogram
+     * counts are added atomically, so every result is the serial one */
+    #pragma omp parallel reduction(|:failed)
+    {
     double* m = (double*)malloc(sizeof(double) * (size_t)(p > 0 ? p : 1));
-    if (!m) return -1;
-
+    if (!m) failed = 1;
+    #pragma omp for schedule(static)
     for (int64_t b = 0; b < nb; ++b) {
+        if (!m) continue;
         const int64_t o = b * p;
         if (hist_mode == 2) {
             double amax = 0.0;
@@ -136,7 +152,10 @@ int oracle_step(int64_t n, int64_t p, float* theta, const uint16_t* grad,
                 for (int64_t i = 0; i < p; ++i) {
                     float x = (float)bf16_to_double(grad[o + i]) / a32;
                     int64_t bi = oracle_bin(x, bins);
-                    if (bi >= 0) hist[bi] += 1;
+                    if (bi >= 0) {
+                        #pragma omp atomic
+                        hist[bi] += 1;
+                    }
                 }
             }
             continue;
@@ -166,7 +185,10 @@ int oracle_step(int64_t n, int64_t p, float* theta, const uint16_t* grad,
                 codes[o + i] = (uint8_t)nearest_level(x, cb_enc, k);
                 if (hist_mode == 1) {
                     int64_t bi = oracle_bin((float)x, bins);
-                    if (bi >= 0) hist[bi] += 1;
+                    if (bi >= 0) {
+                        #pragma omp atomic
+                        hist[bi] += 1;
+                    }
                 }
             }
         } else {
@@ -176,7 +198,8 @@ int oracle_step(int64_t n, int64_t p, float* theta, const uint16_t* grad,
         s[b] = (float)smax;
     }
     free(m);
-    return 0;
+    }
+    return failed ? -1 : 0;
 }
 
 /* Momenta (unquantised) of one step, for margin checks: m_i as in

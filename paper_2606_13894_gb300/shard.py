@@ -120,10 +120,19 @@ class RankShard:
 
     def __init__(self, tensors: Sequence[Tuple[int, int]], rank: int, world: int, device, *,
                  levels: int = 256, bins: int = 4096, refit_every: int = 10, group=None,
-                 reduce: Optional[Callable[[torch.Tensor], torch.Tensor]] = None):
+                 reduce: Optional[Callable[[torch.Tensor], torch.Tensor]] = None,
+                 split: Optional[Callable[[int], bool]] = None):
         self.pieces = partition(tensors, world)[rank]
         self.entries, self.numel_arena, self.nblocks = local_entries(self.pieces)
         self.table = G.tensor_table(self.entries)
+        # a step makes one gefen_step call per table: with `split`, the pieces
+        # whose period it accepts, then the rest (the same step, in two calls)
+        if split is None:
+            self.call_entries = [self.entries]
+        else:
+            self.call_entries = [x for x in ([e for e in self.entries if split(e[2])],
+                                             [e for e in self.entries if not split(e[2])]) if x]
+        self.tables = [G.tensor_table(x) for x in self.call_entries] or [self.table]
         self.device = torch.device(device)
         self.levels, self.bins, self.refit_every = levels, bins, refit_every
         self.reduce = reduce if reduce is not None else (lambda h: all_reduce_histogram(h, group))
@@ -132,13 +141,19 @@ class RankShard:
         self.codes = torch.zeros(self.numel_arena, dtype=torch.uint8, device=dev)
         self.v = torch.zeros(self.nblocks, dtype=torch.float32, device=dev)
         self.scale = torch.zeros(self.nblocks, dtype=torch.float32, device=dev)
-        self.hist = torch.zeros(bins, dtype=torch.int64, device=dev)
         self.cb = torch.empty(levels, dtype=torch.float32, device=dev)
         self.cb_new = torch.empty(levels, dtype=torch.float32, device=dev)
-        self.ws = G.workspace(G.gefen_step_workspace_size(self.table, G.GEFEN_HIST), dev)
-        self.rws = G.workspace(G.gefen_refit_workspace_size(bins, levels), dev)
+        self.ws = G.workspace(max(G.gefen_step_workspace_size(t, G.GEFEN_HIST) for t in [self.table] + self.tables),
+                              dev)
+        self.set_refit_bins(bins)
         self.t = 0
         self.switch = False
+
+    def set_refit_bins(self, bins: int):
+        """Histogram cells of the following refits (and their DP workspace)."""
+        self.bins = bins
+        self.hist = torch.zeros(bins, dtype=torch.int64, device=self.device)
+        self.rws = G.workspace(G.gefen_refit_workspace_size(bins, self.levels), self.device)
 
     @property
     def numel(self) -> int:
@@ -147,6 +162,15 @@ class RankShard:
     def views(self, arena: torch.Tensor):
         """Views of each piece inside a tensor laid out like this rank's arena."""
         return [arena[o:o + n] for (o, n, _, _) in self.entries]
+
+    def gather(self, per_tensor_flat: Callable[[int], torch.Tensor], dtype, out: Optional[torch.Tensor] = None):
+        """This rank's arena of a model-wide quantity: per_tensor_flat(i) is
+        tensor i flattened; each piece's part is copied to its place."""
+        if out is None:
+            out = torch.zeros(self.numel_arena, dtype=dtype, device=self.device)
+        for pc, (o, n, _, _) in zip(self.pieces, self.entries):
+            out[o:o + n].copy_(per_tensor_flat(pc.tensor)[pc.first_element:pc.first_element + n])
+        return out
 
     def init_codebook(self, grads: torch.Tensor, hp):
         """Algorithm 3 on the first gradient: every rank counts g / block
@@ -169,17 +193,22 @@ class RankShard:
             self.refit_codebook(stream=stream)
         return refit
 
-    def step_local(self, grads: torch.Tensor, hp, stream=None) -> bool:
+    def step_local(self, grads: torch.Tensor, hp, stream=None,
+                   after_call: Optional[Callable[[int], None]] = None) -> bool:
         """The step of this rank's blocks alone; on a refit step it also
-        counts the rank's x = m / s' into self.hist (zeroed first)."""
+        counts the rank's x = m / s' into self.hist (zeroed first).
+        after_call(i) runs after the i-th gefen_step call is enqueued."""
         self.t += 1
         refit = self.refit_every > 0 and self.t % self.refit_every == 0
         enc = self.cb_new if self.switch else self.cb
         if refit:
             self.hist.zero_()
-        G.gefen_step(self.table, self.theta, grads, self.codes, self.v, self.scale, self.cb, enc, step=self.t,
-                     flags=G.GEFEN_HIST if refit else 0, hist=self.hist if refit else None,
-                     workspace_buf=self.ws, stream=stream, **hp)
+        for i, tb in enumerate(self.tables):
+            G.gefen_step(tb, self.theta, grads, self.codes, self.v, self.scale, self.cb, enc, step=self.t,
+                         flags=G.GEFEN_HIST if refit else 0, hist=self.hist if refit else None,
+                         workspace_buf=self.ws, stream=stream, **hp)
+            if after_call is not None:
+                after_call(i)
         if self.switch:
             self.cb.copy_(self.cb_new)
             self.switch = False

@@ -1,6 +1,7 @@
-"""The bench's multi-rank path on CPU: replicas with no data-path collective,
-the job time is the slowest rank's, the value counts every rank's parameters,
-and under torchrun only rank 0 prints the reference arm's line."""
+"""The bench's multi-rank path on CPU: the job time is the slowest rank's, the
+value is the model's parameters per second over that time (the ranks share
+one block-sharded model), and under torchrun only rank 0 prints the reference
+arm's line."""
 import json
 import os
 import socket
@@ -30,7 +31,7 @@ def _rank(rank, world, port, q):
     try:
         local_ms = [120.0, 80.0][rank]
         job = bench.job_time_ms(local_ms, world, torch.device("cpu"))
-        q.put((rank, job, bench.whole_job_value(1000, world, 10, job)))
+        q.put((rank, job, bench.whole_job_value(1000, 10, job)))
     finally:
         dist.destroy_process_group()
 
@@ -48,8 +49,8 @@ def test_job_time_is_the_slowest_rank_and_value_counts_all_ranks():
     got = sorted(q.get(timeout=5) for _ in range(2))
     for _, job, value in got:
         assert job == 120.0
-        # 2 ranks x 1000 params x 10 steps in 0.12 s
-        assert value == pytest.approx(2 * 1000 * 10 / 0.12 / 1e9)
+        # a 1000-parameter model, 10 steps in 0.12 s
+        assert value == pytest.approx(1000 * 10 / 0.12 / 1e9)
 
 
 def test_single_rank_needs_no_process_group():
