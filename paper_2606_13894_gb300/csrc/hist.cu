@@ -3,11 +3,16 @@
 //
 // HBM-bound: 4 bytes read per value.  Counts are privatised in shared memory
 // and flushed to the u64 result once per CTA.  Up to 16384 cells: u32
-// counters.  Up to 65536 cells: two 16-bit counters per u32 word (128 KB for
-// 65536 cells, one CTA per SM), kept below 2^16 by construction: after every
-// kPackedUnits units (at most 49152 values) the CTA moves each counter that
-// has reached 2^14 to the u64 result, so between checks none can pass
-// 2^14 - 1 + 49152 = 65535.  NaN values are skipped.
+// counters, two CTAs per SM.  Up to 65536 cells, one CTA per SM: u32 counters
+// for the (at most 49152) central cells, where normalised momentum piles up,
+// and two 16-bit counters per u32 word for the outer ones (224 KB at 65536
+// cells), kept below 2^16 by construction: after every kPackedUnits units (at
+// most 49152 values) the CTA moves each outer counter that has reached 2^14
+// to the u64 result, so between checks none can pass 2^14 - 1 + 49152 =
+// 65535.  That path computes a cell in seven instructions (a round-down add of
+// 1.5 * 2^23 takes the floor), lets a warp whose 512 values of a round share
+// one cell count them with a single atomic, and asks L2 for its next units
+// ahead of the loads.  NaN values are skipped.
 #include <algorithm>
 #include <vector>
 
@@ -22,7 +27,6 @@ constexpr int kHistThreads = 1024;
 constexpr int kHistMaxRanges = 512;
 constexpr int64_t kHistUnit = 16384;  // values per work unit
 constexpr int kHistLoads = 4;         // float4 loads in flight per thread
-constexpr int kPacked = 16;           // hist_body mode: two 16-bit counters per word
 constexpr int kPackedUnits = 3;       // units between checks of the 16-bit counters
 constexpr unsigned kSpillAt = 1u << 14;
 
@@ -44,43 +48,15 @@ __device__ __forceinline__ int find_range(const HistLaunch& L, int64_t unit) {
     return lo;
 }
 
-template <int CL>
 __device__ __forceinline__ void count_one(float x, float halfB, int B, unsigned* local) {
     if (isnan(x)) return;
-    const int c = hist_cell(x, halfB, B);
-    if (CL == kPacked)
-        atomicAdd(local + (c >> 1), 1u << ((c & 1) << 4));  // cell c: half c & 1 of word c / 2
-    else
-        atomicAdd(local + c, 1u);
+    atomicAdd(local + hist_cell(x, halfB, B), 1u);
 }
 
-// Moves every 16-bit counter that has reached kSpillAt to the u64 result
-// (between two CTA barriers: no count is in flight).
-__device__ __forceinline__ void spill_packed(unsigned* words, int B, uint64_t* __restrict__ hist) {
-    const int nw = (B + 1) >> 1;
-    for (int i = threadIdx.x; i < nw; i += blockDim.x) {
-        const unsigned w = words[i];
-        const unsigned lo = w & 0xFFFFu, hi = w >> 16;
-        if (lo < kSpillAt && hi < kSpillAt) continue;
-        unsigned keep = w;
-        if (lo >= kSpillAt) {
-            atomicAdd(reinterpret_cast<unsigned long long*>(hist + 2 * i), static_cast<unsigned long long>(lo));
-            keep &= 0xFFFF0000u;
-        }
-        if (hi >= kSpillAt) {
-            atomicAdd(reinterpret_cast<unsigned long long*>(hist + 2 * i + 1), static_cast<unsigned long long>(hi));
-            keep &= 0x0000FFFFu;
-        }
-        words[i] = keep;
-    }
-}
-
-template <int CL>
 __device__ __forceinline__ void hist_body(const float* __restrict__ x, const HistLaunch& L,
                                           uint64_t* __restrict__ hist, unsigned* s_hist) {
     const int B = L.bins;
     const float halfB = 0.5f * static_cast<float>(B);
-    int since = 0;  // units since the last check of the 16-bit counters (uniform)
     for (int64_t u = blockIdx.x; u < L.nunits; u += gridDim.x) {
         const int r = find_range(L, u);
         const int64_t s0 = L.off[r] + (u - L.unit_begin[r]) * kHistUnit;
@@ -90,7 +66,7 @@ __device__ __forceinline__ void hist_body(const float* __restrict__ x, const His
         int64_t h = (s0 + 3) & ~int64_t(3);
         if (h > s1) h = s1;
         for (int64_t e = s0 + threadIdx.x; e < h; e += blockDim.x)
-            count_one<CL>(__ldcg(x + e), halfB, B, s_hist);
+            count_one(__ldcg(x + e), halfB, B, s_hist);
         const int64_t nv = (s1 - h) >> 2;
         const float4* xv = reinterpret_cast<const float4*>(x + h);
         // kHistLoads float4 loads in flight per thread before any count (a
@@ -104,20 +80,14 @@ __device__ __forceinline__ void hist_body(const float* __restrict__ x, const His
             }
 #pragma unroll
             for (int u = 0; u < kHistLoads; ++u) {
-                count_one<CL>(q[u].x, halfB, B, s_hist);
-                count_one<CL>(q[u].y, halfB, B, s_hist);
-                count_one<CL>(q[u].z, halfB, B, s_hist);
-                count_one<CL>(q[u].w, halfB, B, s_hist);
+                count_one(q[u].x, halfB, B, s_hist);
+                count_one(q[u].y, halfB, B, s_hist);
+                count_one(q[u].z, halfB, B, s_hist);
+                count_one(q[u].w, halfB, B, s_hist);
             }
         }
         for (int64_t e = h + nv * 4 + threadIdx.x; e < s1; e += blockDim.x)
-            count_one<CL>(__ldcg(x + e), halfB, B, s_hist);
-        if (CL == kPacked && ++since == kPackedUnits) {
-            since = 0;
-            __syncthreads();
-            spill_packed(s_hist, B, hist);
-            __syncthreads();
-        }
+            count_one(__ldcg(x + e), halfB, B, s_hist);
     }
 }
 
@@ -127,7 +97,7 @@ __global__ void __launch_bounds__(kHistThreads) k_hist1(const float* __restrict_
     const int B = L.bins;
     for (int i = threadIdx.x; i < B; i += blockDim.x) s_hist[i] = 0u;
     __syncthreads();
-    hist_body<1>(x, L, hist, s_hist);
+    hist_body(x, L, hist, s_hist);
     __syncthreads();
     for (int i = threadIdx.x; i < B; i += blockDim.x) {
         const unsigned c = s_hist[i];
@@ -135,22 +105,201 @@ __global__ void __launch_bounds__(kHistThreads) k_hist1(const float* __restrict_
     }
 }
 
-__global__ void __launch_bounds__(kHistThreads) k_hist16(const float* __restrict__ x,
-                                                        const __grid_constant__ HistLaunch L,
-                                                        uint64_t* __restrict__ hist) {
-    extern __shared__ unsigned s_words[];  // cell c: half c & 1 of word c / 2
-    const int B = L.bins;
-    const int nw = (B + 1) >> 1;
-    for (int i = threadIdx.x; i < nw; i += blockDim.x) s_words[i] = 0u;
-    __syncthreads();
-    hist_body<kPacked>(x, L, hist, s_words);
-    __syncthreads();
-    for (int i = threadIdx.x; i < nw; i += blockDim.x) {
-        const unsigned w = s_words[i];
+// ------------------------------------------------- 16-bit counter path
+// Cells of the 65536-cell path as the bits of a float: t = x + 1 and
+// u = t * (B/2), each rounded to nearest as the cell definition fixes, clamped
+// to [0, B-1] in fp32, then floored by one round-down add of 1.5 * 2^23, so
+// that the sum's bits minus kMagicBits are the cell (u < 2^22 here).  NaN maps
+// to kNoCell.
+constexpr float kMagic = 12582912.0f;  // 1.5 * 2^23
+constexpr uint32_t kMagicBits = 0x4B400000u;
+constexpr uint32_t kNoCell = 0xFFFFFFFFu;
+
+__device__ __forceinline__ uint32_t cell_bits(float x, float halfB, float top) {
+    const float u = __fmul_rn(__fadd_rn(x, 1.0f), halfB);
+    const float f = __fadd_rd(fminf(fmaxf(u, 0.0f), top), kMagic);
+    return isnan(x) ? kNoCell : __float_as_uint(f);
+}
+
+// Counters of the 16384 < B <= 65536 path: the ncen central cells
+// [c_lo, c_lo + ncen) have u32 counters (ncen <= 49152: 192 KB); the at most
+// 16384 outer cells share u32 words two at a time as 16-bit counters (outer
+// index o: the cells below c_lo first, then those above the central run).
+// Normalised momentum piles up near 0, so most counts go to u32 counters,
+// which need no overflow checks and take a constant increment.
+struct Cells {
+    unsigned* cen;
+    unsigned* outer;  // outer index o: half o & 1 of word o / 2
+    uint32_t c_lo, ncen;
+};
+
+constexpr uint32_t kMaxCentral = 49152;
+
+// Adds n counts to cell (bits) c.
+__device__ __forceinline__ void count_bits(const Cells& S, uint32_t c, unsigned n) {
+    const uint32_t ci = c - kMagicBits, d = ci - S.c_lo;
+    if (d < S.ncen) {
+        atomicAdd(S.cen + d, n);
+    } else {
+        const uint32_t o = ci < S.c_lo ? ci : ci - S.ncen;
+        atomicAdd(S.outer + (o >> 1), n << ((o & 1u) << 4));
+    }
+}
+
+// Cell of outer index o.
+__device__ __forceinline__ int outer_cell(const Cells& S, uint32_t o) {
+    return static_cast<int>(o < S.c_lo ? o : o + S.ncen);
+}
+
+// Moves every outer 16-bit counter that has reached kSpillAt to the u64
+// result; four words are tested at once and only words with a counter at or
+// above 2^14 are touched (between two CTA barriers: no count is in flight).
+__device__ __forceinline__ void spill_packed4(const Cells& S, int nw, uint64_t* __restrict__ hist) {
+    static_assert(kSpillAt == (1u << 14), "the test below looks at bits 14 and 15");
+    unsigned* words = S.outer;
+    auto one = [&](int i) {
+        const unsigned w = words[i];
         const unsigned lo = w & 0xFFFFu, hi = w >> 16;
-        if (lo) atomicAdd(reinterpret_cast<unsigned long long*>(hist + 2 * i), static_cast<unsigned long long>(lo));
-        if (hi && 2 * i + 1 < B)
-            atomicAdd(reinterpret_cast<unsigned long long*>(hist + 2 * i + 1), static_cast<unsigned long long>(hi));
+        unsigned keep = w;
+        if (lo >= kSpillAt) {
+            atomicAdd(reinterpret_cast<unsigned long long*>(hist + outer_cell(S, 2 * i)),
+                      static_cast<unsigned long long>(lo));
+            keep &= 0xFFFF0000u;
+        }
+        if (hi >= kSpillAt) {
+            atomicAdd(reinterpret_cast<unsigned long long*>(hist + outer_cell(S, 2 * i + 1)),
+                      static_cast<unsigned long long>(hi));
+            keep &= 0x0000FFFFu;
+        }
+        if (keep != w) words[i] = keep;
+    };
+    const uint4* w4 = reinterpret_cast<const uint4*>(words);
+    for (int i = threadIdx.x; i < (nw >> 2); i += blockDim.x) {
+        const uint4 a = w4[i];
+        if (((a.x | a.y | a.z | a.w) & 0xC000C000u) == 0u) continue;
+        one(4 * i);
+        one(4 * i + 1);
+        one(4 * i + 2);
+        one(4 * i + 3);
+    }
+    for (int i = (nw & ~3) + static_cast<int>(threadIdx.x); i < nw; i += blockDim.x) one(i);
+}
+
+// Asks L2 to fetch the 16-byte aligned body of unit u (no registers or
+// shared memory held while it is in flight).
+__device__ __forceinline__ void prefetch_unit_l2(const float* __restrict__ x, const HistLaunch& L, int64_t u) {
+    const int r = find_range(L, u);
+    const int64_t s0 = L.off[r] + (u - L.unit_begin[r]) * kHistUnit;
+    const int64_t s1 = min(s0 + kHistUnit, L.off[r] + L.cnt[r]);
+    const int64_t h = (s0 + 3) & ~int64_t(3);
+    if (s1 - h < 4) return;
+    const uint32_t bytes = static_cast<uint32_t>(((s1 - h) >> 2) * 16);
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(x + h), "r"(bytes) : "memory");
+}
+
+constexpr int kPrefetchUnits = 2;  // units of this CTA ahead of the one it counts
+
+// 16384 < B <= 65536 cells (Cells: u32 central counters, 16-bit outer pairs;
+// 224 KB at 65536 cells, one CTA per SM).  Shared memory leaves room for no
+// second CTA, so the loads in flight come from L2: thread 0 asks L2 for this
+// CTA's unit kPrefetchUnits ahead while the CTA counts, and each thread keeps
+// four 16-byte loads in flight.  When all 512 values of a warp's round fall in
+// one cell (or are all NaN) the warp adds them with one atomic, else every
+// value is one atomic.  After every kPackedUnits units (at most 49152 values)
+// the CTA moves each outer counter that has reached 2^14 to the u64 result,
+// so none can pass 2^14 - 1 + 49152 = 65535 and carry into its neighbour.
+__global__ void __launch_bounds__(kHistThreads, 1) k_hist16(const float* __restrict__ x,
+                                                           const __grid_constant__ HistLaunch L,
+                                                           uint64_t* __restrict__ hist) {
+    extern __shared__ uint4 s_dyn[];
+    const int B = L.bins;
+    Cells S;
+    S.ncen = min(static_cast<uint32_t>(B), kMaxCentral);
+    S.c_lo = (static_cast<uint32_t>(B) - S.ncen) / 2;
+    S.cen = reinterpret_cast<unsigned*>(s_dyn);
+    S.outer = S.cen + S.ncen;  // ncen is a multiple of 4 or B itself (no outer cells)
+    const int nw = static_cast<int>((static_cast<uint32_t>(B) - S.ncen + 1) >> 1);
+    for (int i = threadIdx.x; i < static_cast<int>(S.ncen) + nw; i += blockDim.x) S.cen[i] = 0u;
+    if (threadIdx.x == 0)
+        for (int p = 0; p < kPrefetchUnits; ++p) {
+            const int64_t u = blockIdx.x + static_cast<int64_t>(p) * gridDim.x;
+            if (u < L.nunits) prefetch_unit_l2(x, L, u);
+        }
+    __syncthreads();
+    const float halfB = 0.5f * static_cast<float>(B), top = static_cast<float>(B - 1);
+    const int lane = threadIdx.x & 31;
+    int since = 0;  // units since the last check of the counters (uniform)
+    for (int64_t u = blockIdx.x; u < L.nunits; u += gridDim.x) {
+        if (threadIdx.x == 0) {
+            const int64_t un = u + static_cast<int64_t>(kPrefetchUnits) * gridDim.x;
+            if (un < L.nunits) prefetch_unit_l2(x, L, un);
+        }
+        const int r = find_range(L, u);
+        const int64_t s0 = L.off[r] + (u - L.unit_begin[r]) * kHistUnit;
+        const int64_t s1 = min(s0 + kHistUnit, L.off[r] + L.cnt[r]);
+        if (s0 < s1) {
+            // 16-byte aligned body with float4 loads; scalar head and tail
+            int64_t h = (s0 + 3) & ~int64_t(3);
+            if (h > s1) h = s1;
+            for (int64_t e = s0 + threadIdx.x; e < h; e += blockDim.x) {
+                const uint32_t c = cell_bits(__ldcg(x + e), halfB, top);
+                if (c != kNoCell) count_bits(S, c, 1u);
+            }
+            const int64_t nv = (s1 - h) >> 2;
+            const float4* xv = reinterpret_cast<const float4*>(x + h);
+            for (int64_t jw = threadIdx.x & ~31; jw < nv; jw += kHistLoads * blockDim.x) {
+                float4 q[kHistLoads];
+#pragma unroll
+                for (int k = 0; k < kHistLoads; ++k) {
+                    const int64_t j = jw + lane + static_cast<int64_t>(k) * blockDim.x;
+                    q[k] = j < nv ? __ldcg(xv + j) : make_float4(NAN, NAN, NAN, NAN);
+                }
+                uint32_t c[4 * kHistLoads];
+#pragma unroll
+                for (int k = 0; k < kHistLoads; ++k) {
+                    c[4 * k] = cell_bits(q[k].x, halfB, top);
+                    c[4 * k + 1] = cell_bits(q[k].y, halfB, top);
+                    c[4 * k + 2] = cell_bits(q[k].z, halfB, top);
+                    c[4 * k + 3] = cell_bits(q[k].w, halfB, top);
+                }
+                uint32_t diff = 0;
+#pragma unroll
+                for (int k = 1; k < 4 * kHistLoads; ++k) diff |= c[k] ^ c[0];
+                const uint32_t c0 = __shfl_sync(0xffffffffu, c[0], 0);
+                if (__all_sync(0xffffffffu, diff == 0u && c[0] == c0)) {
+                    if (lane == 0 && c0 != kNoCell) count_bits(S, c0, 32u * 4u * kHistLoads);
+                } else {
+#pragma unroll
+                    for (int k = 0; k < 4 * kHistLoads; ++k)
+                        if (c[k] != kNoCell) count_bits(S, c[k], 1u);
+                }
+            }
+            for (int64_t e = h + nv * 4 + threadIdx.x; e < s1; e += blockDim.x) {
+                const uint32_t c = cell_bits(__ldcg(x + e), halfB, top);
+                if (c != kNoCell) count_bits(S, c, 1u);
+            }
+        }
+        if (++since == kPackedUnits) {
+            since = 0;
+            __syncthreads();
+            spill_packed4(S, nw, hist);
+            __syncthreads();
+        }
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < static_cast<int>(S.ncen); i += blockDim.x) {
+        const unsigned c = S.cen[i];
+        if (c) atomicAdd(reinterpret_cast<unsigned long long*>(hist + S.c_lo + i), static_cast<unsigned long long>(c));
+    }
+    const uint32_t nouter = static_cast<uint32_t>(B) - S.ncen;
+    for (int i = threadIdx.x; i < nw; i += blockDim.x) {
+        const unsigned w = S.outer[i];
+        const unsigned lo = w & 0xFFFFu, hi = w >> 16;
+        if (lo) atomicAdd(reinterpret_cast<unsigned long long*>(hist + outer_cell(S, 2 * i)),
+                          static_cast<unsigned long long>(lo));
+        if (hi && static_cast<uint32_t>(2 * i + 1) < nouter)
+            atomicAdd(reinterpret_cast<unsigned long long*>(hist + outer_cell(S, 2 * i + 1)),
+                      static_cast<unsigned long long>(hi));
     }
 }
 
@@ -198,7 +347,9 @@ cudaError_t launch_histogram(const float* x, const HistRange* ranges, int nrange
             const int64_t grid = std::min<int64_t>(units, 2 * static_cast<int64_t>(sms));
             k_hist1<<<dim3(static_cast<unsigned>(grid)), kHistThreads, smem, stream>>>(x, L, hist);
         } else {
-            const size_t smem = static_cast<size_t>((bins + 1) / 2) * sizeof(unsigned);
+            // u32 counters for up to 49152 central cells, 16-bit pairs for the rest
+            const size_t ncen = std::min<size_t>(bins, 49152);
+            const size_t smem = (ncen + (bins - ncen + 1) / 2) * sizeof(unsigned);
             e = cudaFuncSetAttribute(k_hist16, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
             if (e != cudaSuccess) return e;
             // resident CTAs per SM for this size (asked once per size)

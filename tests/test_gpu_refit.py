@@ -31,8 +31,11 @@ def _refit_from_hist(h, k):
 def test_histogram_bit_exact(bins, n):
     rng = np.random.default_rng(n + bins)
     x = np.clip(rng.standard_t(4, n) / 8, -1.2, 1.2).astype(np.float32)
-    if n > 10:
+    if n > 20:
         x[:6] = [-1.0, 1.0, 0.0, np.nan, -0.0, np.float32(-1.0 + 2.0 / bins)]
+        # outside [-1, 1] (clamped to the end cells) and next to a cell edge
+        x[6:14] = [np.inf, -np.inf, 1e30, -1e30, 1.5, -3.0, np.nextafter(np.float32(1), np.float32(0)),
+                   np.nextafter(np.float32(-1), np.float32(0))]
     xd = torch.from_numpy(x).cuda()
     ho = torch.zeros(bins, dtype=torch.int64, device="cuda")
     cbo = torch.empty(4, dtype=torch.float32, device="cuda")
@@ -59,6 +62,30 @@ def test_histogram_one_cell(bins, offset):
     ref = oracle.histogram(x[offset:], bins)
     assert ref.max() == n
     np.testing.assert_array_equal(ho.cpu().numpy().astype(np.uint64), ref)
+
+
+@pytest.mark.parametrize("bins", [65536, 40000])
+def test_histogram_runs_of_one_cell(bins):
+    # runs of 512 to 4096 equal values (a warp round whose values share one
+    # cell is counted by one atomic) between random values, NaN runs, and a
+    # start that is not a multiple of four values
+    rng = np.random.default_rng(bins)
+    parts = []
+    for _ in range(3000):
+        m = int(rng.integers(1, 9)) * 512
+        kind = rng.integers(3)
+        if kind == 0:
+            parts.append(np.full(m, rng.uniform(-1, 1), np.float32))
+        elif kind == 1:
+            parts.append(rng.uniform(-1, 1, int(rng.integers(1, 700))).astype(np.float32))
+        else:
+            parts.append(np.full(m, np.nan, np.float32))
+    x = np.concatenate([np.zeros(3, np.float32)] + parts)
+    xd = torch.from_numpy(x).cuda()[4:]  # 16-byte aligned start past the first values
+    ho = torch.zeros(bins, dtype=torch.int64, device="cuda")
+    cbo = torch.empty(4, dtype=torch.float32, device="cuda")
+    G.gefen_refit_codebook(bins=bins, k=4, codebook_out=cbo, x=xd, hist_out=ho)
+    np.testing.assert_array_equal(ho.cpu().numpy().astype(np.uint64), oracle.histogram(x[4:], bins))
 
 
 def test_histogram_input_must_be_16_byte_aligned():
