@@ -147,7 +147,8 @@ gefen_status_t gefen_step(const gefen_tensor_t* tensors, int32_t ntensors,
 
 /* Synchronises `stream` and reports whether a step that used this workspace
  * gave up a bounded wait for its own shared-memory copies (GEFEN_ETIMEOUT; the
- * step's outputs are then not valid).  Reading the flag clears it. */
+ * step's outputs are then not valid).  Reading the flag clears it.  The same
+ * call reads the flag of a gefen_muon_step or gefen_gemm_bf16 workspace. */
 gefen_status_t gefen_step_status(void* workspace, gefen_stream_t stream);
 
 /* -------------------------------------------------------------------------
@@ -291,10 +292,11 @@ gefen_status_t gefen_infer_blocks(const uint16_t* grad, int64_t numel, double ep
  *   theta <- theta (1 - lr weight_decay) - lr sqrt(max(1, rows/cols)) X
  * (Muon as in PyTorch's torch.optim.Muon: momentum 0.95, Nesterov, 5 steps of
  * (3.4445, -4.7750, 2.0315), eps 1e-7 are its defaults).  The matrix
- * products run on cuBLAS: fp32, or with GEFEN_MUON_BF16_GEMM bf16 storage and
- * tensor cores with fp32 accumulation (as Muon runs them).  The first call on
- * a device creates a cuBLAS handle, which allocates its own small state once;
- * the products' scratch comes from the workspace.
+ * products are this library's: with GEFEN_MUON_BF16_GEMM bf16 storage and
+ * fp32 accumulation on the tensor cores (gefen_gemm_bf16, as Muon runs them),
+ * else fp32 throughout on the CUDA cores.  Word 0 of the workspace is set if
+ * a bounded wait of the products gave up (gefen_step_status reads and clears
+ * it; the outputs are then not valid).
  *
  * params f32[rows*cols], grads bf16[rows*cols] (16-byte aligned), codes
  * u8[rows*cols], scale f32[rows*cols/period] (device, in/out); codebooks
@@ -315,6 +317,23 @@ typedef struct {
 } gefen_muon_hparams_t;
 
 size_t gefen_muon_workspace_size(int64_t rows, int64_t cols, int64_t period, uint32_t flags);
+
+/* The product Gefen-Muon's Newton-Schulz iteration runs on (the paper has no
+ * counterpart; exposed for tests and for callers who want it):
+ *   C = alpha * A * B^T + beta * D
+ * A: M x K, B: N x K, C and D: M x N, all row-major bf16 (bit patterns) with
+ * leading dimensions lda >= K, ldb >= K, ldd >= N, ldc >= N; CT (nullable)
+ * receives C transposed (N x M, ldct >= M); C may be NULL when CT is given; D
+ * is read only when beta != 0.  fp32 accumulation; each output rounded once
+ * to bf16.  With 16-byte aligned A and B and lda, ldb multiples of 8 the
+ * product runs on the tensor cores (tcgen05, operands staged by TMA), else on
+ * the CUDA cores.  workspace: >= 256 bytes, 256-byte aligned; its word 0 is
+ * set if a bounded wait gave up (read it with gefen_step_status). */
+gefen_status_t gefen_gemm_bf16(int32_t M, int32_t N, int32_t K, float alpha, const uint16_t* A,
+                               int32_t lda, const uint16_t* B, int32_t ldb, float beta,
+                               const uint16_t* D, int32_t ldd, uint16_t* C, int32_t ldc,
+                               uint16_t* CT, int32_t ldct, void* workspace, size_t workspace_bytes,
+                               gefen_stream_t stream);
 gefen_status_t gefen_muon_step(int64_t rows, int64_t cols, int64_t period, float* params,
                                const uint16_t* grads, uint8_t* codes, float* scale,
                                const float* codebook_dec, const float* codebook_enc, int32_t k,

@@ -1,9 +1,9 @@
 """Build libgefen.so (the C-ABI CUDA library) in-tree for sm_103a.
 
 Each translation unit under ``csrc/`` is compiled in parallel with nvcc, then
-the objects are linked into ``_build/libgefen.so`` (with cuBLAS, for the
-Gefen-Muon products).  The CUDA runtime is linked
-shared so the process uses one runtime together with PyTorch.
+the objects are linked into ``_build/libgefen.so``.  The CUDA runtime is linked
+shared so the process uses one runtime together with PyTorch; the TMA
+tensor-map encoder is taken from the driver at run time.
 """
 from __future__ import annotations
 
@@ -69,7 +69,7 @@ def build(force: bool = False, verbose: bool = False, extra=()) -> str:
     with cf.ThreadPoolExecutor(max_workers=min(8, len(srcs))) as ex:
         objs = list(ex.map(lambda s: _compile(s, list(extra)), srcs))
     tmp = LIB + f".tmp{os.getpid()}"
-    cmd = [nvcc(), *ARCH, "-shared", "-cudart", "shared", "-o", tmp, *objs, "-lcublas"]
+    cmd = [nvcc(), *ARCH, "-shared", "-cudart", "shared", "-o", tmp, *objs]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError("link failed:\n" + r.stderr)

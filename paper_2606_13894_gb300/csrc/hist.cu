@@ -106,44 +106,51 @@ __global__ void __launch_bounds__(kHistThreads) k_hist1(const float* __restrict_
 }
 
 // ------------------------------------------------- 16-bit counter path
-// Cells of the 65536-cell path as the bits of a float: t = x + 1 and
-// u = t * (B/2), each rounded to nearest as the cell definition fixes, clamped
-// to [0, B-1] in fp32, then floored by one round-down add of 1.5 * 2^23, so
-// that the sum's bits minus kMagicBits are the cell (u < 2^22 here).  NaN maps
-// to kNoCell.
+// Cells of the 65536-cell path as the bits of a float: the floor of the cell
+// coordinate is taken by a round-down add of 1.5 * 2^23, so that the sum's
+// bits minus kMagicBits are the cell (coordinates below 2^22 here).  With B a
+// power of two the scaling by B/2 is exact, so RN(x + 1) * B/2 floored by one
+// round-down fma is the cell definition's floor(RN(RN(x + 1) * B/2)), clamped
+// in the integer domain; other B take the definition's two roundings, clamped
+// in fp32.  NaN maps to nan_bits (the trash counter, see Cells).
 constexpr float kMagic = 12582912.0f;  // 1.5 * 2^23
 constexpr uint32_t kMagicBits = 0x4B400000u;
-constexpr uint32_t kNoCell = 0xFFFFFFFFu;
 
-__device__ __forceinline__ uint32_t cell_bits(float x, float halfB, float top) {
-    const float u = __fmul_rn(__fadd_rn(x, 1.0f), halfB);
-    const float f = __fadd_rd(fminf(fmaxf(u, 0.0f), top), kMagic);
-    return isnan(x) ? kNoCell : __float_as_uint(f);
+template <bool POW2>
+__device__ __forceinline__ uint32_t cell_bits(float x, float halfB, float top, int top_bits, uint32_t nan_bits) {
+    uint32_t c;
+    if (POW2) {
+        const float f = __fmaf_rd(__fadd_rn(x, 1.0f), halfB, kMagic);
+        c = static_cast<uint32_t>(max(min(__float_as_int(f), top_bits), static_cast<int>(kMagicBits)));
+    } else {
+        const float u = __fmul_rn(__fadd_rn(x, 1.0f), halfB);
+        c = __float_as_uint(__fadd_rd(fminf(fmaxf(u, 0.0f), top), kMagic));
+    }
+    return isnan(x) ? nan_bits : c;
 }
 
 // Counters of the 16384 < B <= 65536 path: the ncen central cells
 // [c_lo, c_lo + ncen) have u32 counters (ncen <= 49152: 192 KB); the at most
 // 16384 outer cells share u32 words two at a time as 16-bit counters (outer
-// index o: the cells below c_lo first, then those above the central run).
+// index o: the cells below c_lo first, then those above the central run),
+// followed by one trash word that NaN values count into (never read).
 // Normalised momentum piles up near 0, so most counts go to u32 counters,
-// which need no overflow checks and take a constant increment.
+// which need no overflow checks.
 struct Cells {
     unsigned* cen;
-    unsigned* outer;  // outer index o: half o & 1 of word o / 2
+    unsigned* outer;  // outer index o: half o & 1 of word o / 2; word nw: trash
     uint32_t c_lo, ncen;
 };
 
 constexpr uint32_t kMaxCentral = 49152;
 
-// Adds n counts to cell (bits) c.
+// Adds n counts to cell (bits) c, without a branch.
 __device__ __forceinline__ void count_bits(const Cells& S, uint32_t c, unsigned n) {
     const uint32_t ci = c - kMagicBits, d = ci - S.c_lo;
-    if (d < S.ncen) {
-        atomicAdd(S.cen + d, n);
-    } else {
-        const uint32_t o = ci < S.c_lo ? ci : ci - S.ncen;
-        atomicAdd(S.outer + (o >> 1), n << ((o & 1u) << 4));
-    }
+    const bool cen = d < S.ncen;
+    const uint32_t o = ci < S.c_lo ? ci : ci - S.ncen;
+    unsigned* w = cen ? S.cen + d : S.outer + (o >> 1);
+    atomicAdd(w, cen ? n : n << ((o & 1u) << 4));
 }
 
 // Cell of outer index o.
@@ -208,6 +215,7 @@ constexpr int kPrefetchUnits = 2;  // units of this CTA ahead of the one it coun
 // value is one atomic.  After every kPackedUnits units (at most 49152 values)
 // the CTA moves each outer counter that has reached 2^14 to the u64 result,
 // so none can pass 2^14 - 1 + 49152 = 65535 and carry into its neighbour.
+template <bool POW2>
 __global__ void __launch_bounds__(kHistThreads, 1) k_hist16(const float* __restrict__ x,
                                                            const __grid_constant__ HistLaunch L,
                                                            uint64_t* __restrict__ hist) {
@@ -217,9 +225,12 @@ __global__ void __launch_bounds__(kHistThreads, 1) k_hist16(const float* __restr
     S.ncen = min(static_cast<uint32_t>(B), kMaxCentral);
     S.c_lo = (static_cast<uint32_t>(B) - S.ncen) / 2;
     S.cen = reinterpret_cast<unsigned*>(s_dyn);
-    S.outer = S.cen + S.ncen;  // ncen is a multiple of 4 or B itself (no outer cells)
+    S.outer = S.cen + ((S.ncen + 3) & ~3u);  // 16-byte aligned for the four-word spill test
     const int nw = static_cast<int>((static_cast<uint32_t>(B) - S.ncen + 1) >> 1);
-    for (int i = threadIdx.x; i < static_cast<int>(S.ncen) + nw; i += blockDim.x) S.cen[i] = 0u;
+    for (int i = threadIdx.x; i < static_cast<int>((S.ncen + 3) & ~3u) + nw + 1; i += blockDim.x) S.cen[i] = 0u;
+    // NaN: outer index 2 nw, the low half of the trash word
+    const uint32_t nan_bits = kMagicBits + 2u * static_cast<uint32_t>(nw) + S.ncen;
+    const int top_bits = static_cast<int>(kMagicBits) + B - 1;
     if (threadIdx.x == 0)
         for (int p = 0; p < kPrefetchUnits; ++p) {
             const int64_t u = blockIdx.x + static_cast<int64_t>(p) * gridDim.x;
@@ -242,8 +253,8 @@ __global__ void __launch_bounds__(kHistThreads, 1) k_hist16(const float* __restr
             int64_t h = (s0 + 3) & ~int64_t(3);
             if (h > s1) h = s1;
             for (int64_t e = s0 + threadIdx.x; e < h; e += blockDim.x) {
-                const uint32_t c = cell_bits(__ldcg(x + e), halfB, top);
-                if (c != kNoCell) count_bits(S, c, 1u);
+                const uint32_t c = cell_bits<POW2>(__ldcg(x + e), halfB, top, top_bits, nan_bits);
+                count_bits(S, c, 1u);
             }
             const int64_t nv = (s1 - h) >> 2;
             const float4* xv = reinterpret_cast<const float4*>(x + h);
@@ -257,26 +268,25 @@ __global__ void __launch_bounds__(kHistThreads, 1) k_hist16(const float* __restr
                 uint32_t c[4 * kHistLoads];
 #pragma unroll
                 for (int k = 0; k < kHistLoads; ++k) {
-                    c[4 * k] = cell_bits(q[k].x, halfB, top);
-                    c[4 * k + 1] = cell_bits(q[k].y, halfB, top);
-                    c[4 * k + 2] = cell_bits(q[k].z, halfB, top);
-                    c[4 * k + 3] = cell_bits(q[k].w, halfB, top);
+                    c[4 * k] = cell_bits<POW2>(q[k].x, halfB, top, top_bits, nan_bits);
+                    c[4 * k + 1] = cell_bits<POW2>(q[k].y, halfB, top, top_bits, nan_bits);
+                    c[4 * k + 2] = cell_bits<POW2>(q[k].z, halfB, top, top_bits, nan_bits);
+                    c[4 * k + 3] = cell_bits<POW2>(q[k].w, halfB, top, top_bits, nan_bits);
                 }
                 uint32_t diff = 0;
 #pragma unroll
                 for (int k = 1; k < 4 * kHistLoads; ++k) diff |= c[k] ^ c[0];
                 const uint32_t c0 = __shfl_sync(0xffffffffu, c[0], 0);
                 if (__all_sync(0xffffffffu, diff == 0u && c[0] == c0)) {
-                    if (lane == 0 && c0 != kNoCell) count_bits(S, c0, 32u * 4u * kHistLoads);
+                    if (lane == 0) count_bits(S, c0, 32u * 4u * kHistLoads);
                 } else {
 #pragma unroll
-                    for (int k = 0; k < 4 * kHistLoads; ++k)
-                        if (c[k] != kNoCell) count_bits(S, c[k], 1u);
+                    for (int k = 0; k < 4 * kHistLoads; ++k) count_bits(S, c[k], 1u);
                 }
             }
             for (int64_t e = h + nv * 4 + threadIdx.x; e < s1; e += blockDim.x) {
-                const uint32_t c = cell_bits(__ldcg(x + e), halfB, top);
-                if (c != kNoCell) count_bits(S, c, 1u);
+                const uint32_t c = cell_bits<POW2>(__ldcg(x + e), halfB, top, top_bits, nan_bits);
+                count_bits(S, c, 1u);
             }
         }
         if (++since == kPackedUnits) {
@@ -308,7 +318,8 @@ __global__ void __launch_bounds__(kHistThreads, 1) k_hist16(const float* __restr
 cudaError_t prepare_histogram() {
     cudaFuncAttributes fa;
     cudaError_t e = cudaFuncGetAttributes(&fa, k_hist1);
-    if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, k_hist16);
+    if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, k_hist16<true>);
+    if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, k_hist16<false>);
     return e;
 }
 
@@ -347,16 +358,19 @@ cudaError_t launch_histogram(const float* x, const HistRange* ranges, int nrange
             const int64_t grid = std::min<int64_t>(units, 2 * static_cast<int64_t>(sms));
             k_hist1<<<dim3(static_cast<unsigned>(grid)), kHistThreads, smem, stream>>>(x, L, hist);
         } else {
-            // u32 counters for up to 49152 central cells, 16-bit pairs for the rest
+            // u32 counters for up to 49152 central cells, 16-bit pairs for the
+            // rest, one trash word
             const size_t ncen = std::min<size_t>(bins, 49152);
-            const size_t smem = (ncen + (bins - ncen + 1) / 2) * sizeof(unsigned);
-            e = cudaFuncSetAttribute(k_hist16, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+            const size_t smem = ((ncen + 3) / 4 * 4 + (bins - ncen + 1) / 2 + 1) * sizeof(unsigned);
+            const bool pow2 = (bins & (bins - 1)) == 0;
+            auto k16 = pow2 ? k_hist16<true> : k_hist16<false>;
+            e = cudaFuncSetAttribute(k16, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
             if (e != cudaSuccess) return e;
             // resident CTAs per SM for this size (asked once per size)
             static thread_local size_t fit_smem = 0;
             static thread_local int per_sm = 1;
             if (fit_smem != smem) {
-                if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_hist16, kHistThreads, smem) !=
+                if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k16, kHistThreads, smem) !=
                         cudaSuccess || per_sm < 1) {
                     (void)cudaGetLastError();
                     per_sm = 1;
@@ -364,7 +378,7 @@ cudaError_t launch_histogram(const float* x, const HistRange* ranges, int nrange
                 fit_smem = smem;
             }
             const int64_t grid = std::min<int64_t>(units, static_cast<int64_t>(per_sm) * sms);
-            k_hist16<<<dim3(static_cast<unsigned>(grid)), kHistThreads, smem, stream>>>(x, L, hist);
+            k16<<<dim3(static_cast<unsigned>(grid)), kHistThreads, smem, stream>>>(x, L, hist);
         }
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;

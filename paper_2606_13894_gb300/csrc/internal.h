@@ -27,6 +27,19 @@ cudaError_t launch_histogram(const float* x, const HistRange* ranges, int nrange
 // needs nothing more from the driver).
 cudaError_t prepare_histogram();
 
+// C = alpha * A * B^T + beta * D (row-major; A: M x K, B: N x K, C, D: M x N),
+// written as C and/or as its transpose CT (N x M); bf16 storage with fp32
+// accumulation (tcgen05 when TMA can address A and B), or fp32 throughout.
+// D, C, CT nullable.  err: device word set when a bounded wait gave up.
+cudaError_t gemm_bf16_nt(int M, int N, int K, float alpha, const void* A, int lda, const void* B, int ldb,
+                         float beta, const void* D, int ldd, void* C, int ldc, void* CT, int ldct, int* err,
+                         cudaStream_t st);
+cudaError_t gemm_f32_nt(int M, int N, int K, float alpha, const float* A, int lda, const float* B, int ldb,
+                        float beta, const float* D, int ldd, float* C, int ldc, float* CT, int ldct,
+                        cudaStream_t st);
+// Whether the bf16 product takes the tcgen05 path for these operands.
+bool gemm_tc_usable(int lda, int ldb, const void* A, const void* B);
+
 // Multiprocessor count of the current device (cached per device).
 int device_sm_count();
 

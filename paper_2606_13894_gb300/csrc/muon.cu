@@ -8,15 +8,18 @@
 //   X    = U / max(||U||_F, eps); X <- a X + (b A + c A A) X, A = X X^T,
 //          on the smaller side (ns_steps times)
 //   theta = theta (1 - lr wd) - lr sqrt(max(1, rows/cols)) X
-// The element-wise parts are this file's kernels; the Newton-Schulz products
-// are plain GEMMs on cuBLAS (fp32, or bf16 tensor cores like Muon's own).
+// The element-wise parts and the Newton-Schulz products are this library's
+// kernels: with bf16 storage (as Muon runs them) the products are the tcgen05
+// GEMM of gemm.cu, with fp32 storage its CUDA-core fallback.
 //
-// The row-major rows x cols update buffer is, read column-major, the matrix
-// M = X^T (cols x rows).  With rows <= cols the small side is rows: A = M^T M
-// and M <- M B + a M.  With rows > cols it is cols and M is the transposed
-// working matrix itself: A = M M^T and M <- B M + a M.  No transpose is ever
-// materialised.
-#include <cublas_v2.h>
+// The working matrix X is s x n with s = min(rows, cols) on the small side:
+// X = U for rows <= cols, X = U^T otherwise.  Both X and T = X^T are kept,
+// row-major, so that every product reads K-contiguous operands:
+//   A  = X X^T                      (s x s, K = n)
+//   B  = c A A^T + b A              (A is symmetric: A A^T = A A)
+//   X' = B X + a X = B T^T + a X    (s x n, K = s), written with T' = X'^T
+// One of the two layouts is U's own (rows x cols row-major), so the update
+// reads the result in place.
 #include <cuda_bf16.h>
 
 #include <algorithm>
@@ -32,14 +35,14 @@ namespace {
 
 constexpr int kMuThreads = 256;
 constexpr int kMuPartials = 1024;  // CTAs of the encode kernel (norm partials)
-constexpr size_t kCublasWs = size_t(32) << 20;
 
 struct MuonLayout {
-    size_t hdr, snew, part, m0, m1, ga, gb, cublas, total;
+    size_t hdr, snew, part, p0, p1, q0, q1, ga, gb, total;
 };
 
-// header (256 B) | new scales | norm partials | two update buffers | A | B |
-// cuBLAS workspace
+// header (256 B; word 0: a bounded wait gave up) | new scales | norm
+// partials | two rows x cols buffers (U's layout) | two cols x rows buffers
+// (transposed) | A | B
 MuonLayout muon_layout(int64_t rows, int64_t cols, int64_t period, bool bf16) {
     MuonLayout L;
     const int64_t n = rows * cols, s = std::min(rows, cols);
@@ -48,11 +51,12 @@ MuonLayout muon_layout(int64_t rows, int64_t cols, int64_t period, bool bf16) {
     L.hdr = o; o += kWsAlign;
     L.snew = o; o += align_up(static_cast<size_t>(n / period) * sizeof(float));
     L.part = o; o += align_up(static_cast<size_t>(kMuPartials) * sizeof(double));
-    L.m0 = o; o += align_up(static_cast<size_t>(n) * eb);
-    L.m1 = o; o += align_up(static_cast<size_t>(n) * eb);
+    L.p0 = o; o += align_up(static_cast<size_t>(n) * eb);
+    L.p1 = o; o += align_up(static_cast<size_t>(n) * eb);
+    L.q0 = o; o += align_up(static_cast<size_t>(n) * eb);
+    L.q1 = o; o += align_up(static_cast<size_t>(n) * eb);
     L.ga = o; o += align_up(static_cast<size_t>(s * s) * eb);
     L.gb = o; o += align_up(static_cast<size_t>(s * s) * eb);
-    L.cublas = o; o += kCublasWs;
     L.total = o;
     return L;
 }
@@ -192,25 +196,17 @@ __global__ void __launch_bounds__(kMuThreads) k_muon_update(float* __restrict__ 
     }
 }
 
-// One cuBLAS handle per device, created on first use (cuBLAS keeps its own
-// state; its scratch for our calls comes from the caller's workspace).
-cublasHandle_t muon_handle() {
-    static std::mutex mu;
-    static cublasHandle_t h[64] = {nullptr};
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
-    std::lock_guard<std::mutex> g(mu);
-    if (!h[dev] && cublasCreate(&h[dev]) != CUBLAS_STATUS_SUCCESS) h[dev] = nullptr;
-    return h[dev];
-}
-
-// C = alpha op(A) op(B) + beta C, column-major, fp32 or bf16 storage with fp32
-// accumulation.
-cublasStatus_t gemm(cublasHandle_t h, bool bf16, cublasOperation_t ta, cublasOperation_t tb, int m, int n, int k,
-                    float alpha, const void* A, int lda, const void* B, int ldb, float beta, void* C, int ldc) {
-    const cudaDataType_t ty = bf16 ? CUDA_R_16BF : CUDA_R_32F;
-    return cublasGemmEx(h, ta, tb, m, n, k, &alpha, A, ty, lda, B, ty, ldb, &beta, C, ty, ldc,
-                        CUBLAS_COMPUTE_32F, CUBLAS_GEMM_DEFAULT);
+// out (cols x rows) = in (rows x cols)^T, 32 x 32 tiles through shared memory.
+template <typename T>
+__global__ void __launch_bounds__(256) k_transpose(const T* __restrict__ in, T* __restrict__ out, int rows, int cols) {
+    __shared__ T tile[32][33];
+    const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
+    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+    for (int i = ty; i < 32; i += 8)
+        if (r0 + i < rows && c0 + tx < cols) tile[i][tx] = in[static_cast<int64_t>(r0 + i) * cols + c0 + tx];
+    __syncthreads();
+    for (int i = ty; i < 32; i += 8)
+        if (c0 + i < cols && r0 + tx < rows) out[static_cast<int64_t>(c0 + i) * rows + r0 + tx] = tile[tx][i];
 }
 
 }  // namespace
@@ -245,8 +241,6 @@ extern "C" gefen_status_t gefen_muon_step(int64_t rows, int64_t cols, int64_t pe
     if (workspace == nullptr || workspace_bytes < L.total) return GEFEN_ENOMEM;
     if (reinterpret_cast<uintptr_t>(workspace) % kWsAlign) return GEFEN_EINVAL;
     if (gefen_status_t s = check_device(); s != GEFEN_OK) return s;
-    cublasHandle_t h = muon_handle();
-    if (!h) return GEFEN_ECUDA;
 
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     char* ws = static_cast<char*>(workspace);
@@ -265,11 +259,14 @@ extern "C" gefen_status_t gefen_muon_step(int64_t rows, int64_t cols, int64_t pe
     A.cb_enc = codebook_enc;
     A.snew = reinterpret_cast<float*>(ws + L.snew);
     A.part = reinterpret_cast<double*>(ws + L.part);
-    void* M = ws + L.m0;
-    void* Mn = ws + L.m1;
+    void* P0 = ws + L.p0;
+    void* P1 = ws + L.p1;
+    void* Q0 = ws + L.q0;
+    void* Q1 = ws + L.q1;
     void* GA = ws + L.ga;
     void* GB = ws + L.gb;
-    A.u = M;
+    int* err = reinterpret_cast<int*>(ws + L.hdr);
+    A.u = P0;
 
     const int grid = static_cast<int>(std::min<int64_t>(kMuPartials, (n + kMuThreads - 1) / kMuThreads));
     if (cudaMemsetAsync(A.snew, 0, static_cast<size_t>(n / period) * sizeof(float), st) != cudaSuccess)
@@ -284,41 +281,51 @@ extern "C" gefen_status_t gefen_muon_step(int64_t rows, int64_t cols, int64_t pe
     }
     if (cudaGetLastError() != cudaSuccess) return GEFEN_ECUDA;
 
-    // Newton-Schulz on the column-major view M (cols x rows, ld = cols)
-    if (cublasSetStream(h, st) != CUBLAS_STATUS_SUCCESS ||
-        cublasSetWorkspace(h, ws + L.cublas, kCublasWs) != CUBLAS_STATUS_SUCCESS ||
-        cublasSetMathMode(h, CUBLAS_DEFAULT_MATH) != CUBLAS_STATUS_SUCCESS)
-        return GEFEN_ECUDA;
+    // Newton-Schulz on X (s x n) and T = X^T (n x s): the P buffers hold U's
+    // layout (rows x cols), the Q buffers the transposed one
     const bool wide = rows <= cols;
-    const int s = static_cast<int>(std::min(rows, cols));
-    const int ld = static_cast<int>(cols), nr = static_cast<int>(rows);
-    const size_t eb = bf16 ? 2 : 4;
+    const int s = static_cast<int>(std::min(rows, cols)), nn = static_cast<int>(std::max(rows, cols));
     const float a = static_cast<float>(hp.ns_a), b = static_cast<float>(hp.ns_b), c = static_cast<float>(hp.ns_c);
-    for (int it = 0; it < hp.ns_steps; ++it) {
-        cublasStatus_t cs;
-        // A = X X^T on the small side
-        cs = wide ? gemm(h, bf16, CUBLAS_OP_T, CUBLAS_OP_N, s, s, ld, 1.0f, M, ld, M, ld, 0.0f, GA, s)
-                  : gemm(h, bf16, CUBLAS_OP_N, CUBLAS_OP_T, s, s, nr, 1.0f, M, ld, M, ld, 0.0f, GA, s);
-        if (cs != CUBLAS_STATUS_SUCCESS) return GEFEN_ECUDA;
-        // B = b A + c A A
-        if (cudaMemcpyAsync(GB, GA, static_cast<size_t>(s) * s * eb, cudaMemcpyDeviceToDevice, st) != cudaSuccess)
-            return GEFEN_ECUDA;
-        if (gemm(h, bf16, CUBLAS_OP_N, CUBLAS_OP_N, s, s, s, c, GA, s, GA, s, b, GB, s) != CUBLAS_STATUS_SUCCESS)
-            return GEFEN_ECUDA;
-        // X <- a X + B X  (M <- M B + a M, or M <- B M + a M)
-        if (cudaMemcpyAsync(Mn, M, static_cast<size_t>(n) * eb, cudaMemcpyDeviceToDevice, st) != cudaSuccess)
-            return GEFEN_ECUDA;
-        cs = wide ? gemm(h, bf16, CUBLAS_OP_N, CUBLAS_OP_N, ld, s, s, 1.0f, M, ld, GB, s, a, Mn, ld)
-                  : gemm(h, bf16, CUBLAS_OP_N, CUBLAS_OP_N, s, nr, s, 1.0f, GB, s, M, ld, a, Mn, ld);
-        if (cs != CUBLAS_STATUS_SUCCESS) return GEFEN_ECUDA;
-        std::swap(M, Mn);
+    void* U = P0;
+    if (hp.ns_steps > 0) {
+        const dim3 tg(static_cast<unsigned>((cols + 31) / 32), static_cast<unsigned>((rows + 31) / 32));
+        if (bf16)
+            k_transpose<__nv_bfloat16><<<tg, 256, 0, st>>>(static_cast<const __nv_bfloat16*>(P0),
+                                                           static_cast<__nv_bfloat16*>(Q0), static_cast<int>(rows),
+                                                           static_cast<int>(cols));
+        else
+            k_transpose<float><<<tg, 256, 0, st>>>(static_cast<const float*>(P0), static_cast<float*>(Q0),
+                                                  static_cast<int>(rows), static_cast<int>(cols));
+        void *X = wide ? P0 : Q0, *T = wide ? Q0 : P0, *Xn = wide ? P1 : Q1, *Tn = wide ? Q1 : P1;
+        for (int it = 0; it < hp.ns_steps; ++it) {
+            cudaError_t e;
+            if (bf16) {
+                e = gemm_bf16_nt(s, s, nn, 1.0f, X, nn, X, nn, 0.0f, nullptr, 0, GA, s, nullptr, 0, err, st);
+                if (e == cudaSuccess)
+                    e = gemm_bf16_nt(s, s, s, c, GA, s, GA, s, b, GA, s, GB, s, nullptr, 0, err, st);
+                if (e == cudaSuccess)
+                    e = gemm_bf16_nt(s, nn, s, 1.0f, GB, s, T, s, a, X, nn, Xn, nn, Tn, s, err, st);
+            } else {
+                const float *fx = static_cast<const float*>(X), *ft = static_cast<const float*>(T);
+                float *fa = static_cast<float*>(GA), *fb = static_cast<float*>(GB);
+                e = gemm_f32_nt(s, s, nn, 1.0f, fx, nn, fx, nn, 0.0f, nullptr, 0, fa, s, nullptr, 0, st);
+                if (e == cudaSuccess) e = gemm_f32_nt(s, s, s, c, fa, s, fa, s, b, fa, s, fb, s, nullptr, 0, st);
+                if (e == cudaSuccess)
+                    e = gemm_f32_nt(s, nn, s, 1.0f, fb, s, ft, s, a, fx, nn, static_cast<float*>(Xn), nn,
+                                    static_cast<float*>(Tn), s, st);
+            }
+            if (e != cudaSuccess) return GEFEN_ECUDA;
+            std::swap(X, Xn);
+            std::swap(T, Tn);
+        }
+        U = wide ? X : T;
     }
     const double adj = hp.lr * std::sqrt(std::max(1.0, static_cast<double>(rows) / static_cast<double>(cols)));
     const float decay = static_cast<float>(1.0 - hp.lr * hp.weight_decay);
     if (bf16)
-        k_muon_update<true><<<grid, kMuThreads, 0, st>>>(params, M, n, decay, static_cast<float>(adj));
+        k_muon_update<true><<<grid, kMuThreads, 0, st>>>(params, U, n, decay, static_cast<float>(adj));
     else
-        k_muon_update<false><<<grid, kMuThreads, 0, st>>>(params, M, n, decay, static_cast<float>(adj));
+        k_muon_update<false><<<grid, kMuThreads, 0, st>>>(params, U, n, decay, static_cast<float>(adj));
     if (cudaGetLastError() != cudaSuccess) return GEFEN_ECUDA;
     return GEFEN_OK;
 }

@@ -49,7 +49,7 @@ EXPORTS = ("gefen_status_string", "gefen_sync_status", "gefen_step_workspace_siz
            "gefen_refit_workspace_size", "gefen_refit_codebook", "gefen_refit_status",
            "gefen_refit_tables", "gefen_infer_workspace_size", "gefen_infer_blocks",
            "gefen_refit_codebook_static", "gefen_refit_static_init", "gefen_refit_static_status",
-           "gefen_refit_debug", "gefen_muon_workspace_size", "gefen_muon_step")
+           "gefen_refit_debug", "gefen_muon_workspace_size", "gefen_muon_step", "gefen_gemm_bf16")
 
 GEFEN_MUON_BF16_GEMM = 1
 
@@ -116,6 +116,9 @@ def load(build_if_needed: bool = True):
         L.gefen_muon_workspace_size.restype = sz
         L.gefen_muon_step.argtypes = [i64, i64, i64, P, P, P, P, P, P, i32, gefen_muon_hparams_t, P, sz, P]
         L.gefen_muon_step.restype = ctypes.c_int
+        f32 = ctypes.c_float
+        L.gefen_gemm_bf16.argtypes = [i32, i32, i32, f32, P, i32, P, i32, f32, P, i32, P, i32, P, i32, P, sz, P]
+        L.gefen_gemm_bf16.restype = ctypes.c_int
         _lib = L
         return L
 
@@ -319,3 +322,21 @@ def gefen_muon_step(rows, cols, period, params, grads, codes, scale, codebook_de
                                 _ptr(workspace_buf), workspace_buf.numel(), _stream(stream))
     _check("gefen_muon_step", st)
     return workspace_buf
+
+
+def gefen_gemm_bf16(A, B, *, alpha=1.0, beta=0.0, D=None, C=None, CT=None, workspace_buf=None, stream=None):
+    """C = alpha A B^T + beta D (bf16 row-major tensors; CT gets C transposed).
+    Allocates C when neither C nor CT is given.  Returns (C, CT, workspace)."""
+    M, K = A.shape
+    N = B.shape[0]
+    if C is None and CT is None:
+        C = torch.empty((M, N), dtype=torch.bfloat16, device=A.device)
+    if workspace_buf is None:
+        workspace_buf = workspace(256, A.device)
+    st = load().gefen_gemm_bf16(M, N, K, float(alpha), _ptr(A), A.stride(0), _ptr(B), B.stride(0), float(beta),
+                                _ptr(D), D.stride(0) if D is not None else 0, _ptr(C),
+                                C.stride(0) if C is not None else 0, _ptr(CT),
+                                CT.stride(0) if CT is not None else 0, _ptr(workspace_buf), workspace_buf.numel(),
+                                _stream(stream))
+    _check("gefen_gemm_bf16", st)
+    return C, CT, workspace_buf

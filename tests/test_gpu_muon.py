@@ -60,3 +60,29 @@ def test_muon_step_parity(rows, cols, period, bf16):
         ohp = dict(beta1=hp["momentum"])
         ok, flips = U.code_flips_ok(V, pre, gbits, cb, cb, codes.cpu().numpy(), cd, ohp, Mb)
         assert ok, (t, flips)
+
+
+def test_muon_step_parity_2048x8192_bf16():
+    """The shape the Newton-Schulz timings are quoted on (bf16 products on the
+    tensor cores), one step against the oracle."""
+    rows, cols, period = 2048, 8192, 8192
+    rng = np.random.default_rng(2048)
+    n = rows * cols
+    hp = dict(lr=2e-2, momentum=0.95, weight_decay=0.1, eps=1e-7, nesterov=True)
+    cb = U.codebook(256, rng)
+    theta = torch.from_numpy(rng.normal(0, 0.02, n).astype(np.float32)).cuda()
+    codes = torch.full((n,), U.zero_code(cb), dtype=torch.uint8, device="cuda")
+    s = torch.zeros(n // period, dtype=torch.float32, device="cuda")
+    d_cb = torch.from_numpy(cb).cuda()
+    sig = np.repeat(10 ** rng.uniform(-4, -2, rows), cols)
+    gb = torch.from_numpy((rng.normal(size=n) * sig).astype(np.float32)).to(torch.bfloat16).cuda()
+    gbits = U.bits(gb)
+    th, cd, ss = theta.cpu().numpy().copy(), codes.cpu().numpy().copy(), s.cpu().numpy().copy()
+    ws = G.gefen_muon_step(rows, cols, period, theta, gb, codes, s, d_cb, d_cb, flags=G.GEFEN_MUON_BF16_GEMM, **hp)
+    G.gefen_step_status(ws)
+    X = M.muon_step(th, gbits, cd, ss, cb, cb, rows=rows, cols=cols, period=period, **hp)
+    adj = hp["lr"] * math.sqrt(max(1.0, rows / cols))
+    got = theta.cpu().numpy().astype(np.float64)
+    tol = adj * 6e-2 * np.abs(X).max() + 1e-5 * np.maximum(np.abs(th.astype(np.float64)), hp["lr"])
+    err = np.abs(got - th.astype(np.float64))
+    assert np.all(err <= tol), f"theta off by {float((err / tol).max()):.3g} x tolerance"
