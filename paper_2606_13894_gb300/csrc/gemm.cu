@@ -6,15 +6,18 @@
 // all row-major (K contiguous in A and B), written as C and/or as its
 // transpose CT (N x M).
 //
-// bf16 storage, fp32 accumulation: a tcgen05 kernel.  One CTA computes a
-// 128 x 256 tile of C in tensor memory (256 of its 512 columns).  Thread 0
-// loads 128 x 64 tiles of A and 256 x 64 tiles of B with TMA (128-byte
-// swizzle) into a ring of four shared-memory stages; thread 32 issues
-// tcgen05.mma (M 128, N 256, K 16; four per stage) as each stage lands and
-// frees it with tcgen05.commit; all four warps then read the accumulator rows
-// with tcgen05.ld, apply alpha and beta * D and store C directly, or CT
-// through shared memory so that its rows go out coalesced.  Every wait on an
-// mbarrier gives up after about a second and flags the error word instead.
+// bf16 storage, fp32 accumulation: a persistent tcgen05 kernel, one CTA per
+// SM taking 128 x BN tiles of C (BN 256, or 128 when there are too few
+// tiles).  Warp 0 loads 128 x 64 k-tiles of A and BN x 64 of B with TMA
+// (128-byte swizzle) into a ring of shared-memory stages; warp 1 issues
+// tcgen05.mma (M 128, N BN, K 16; four per stage) into one of two tensor-memory
+// accumulators and frees each stage with tcgen05.commit; warps 2-5 read the
+// other accumulator with tcgen05.ld, apply alpha and beta * D and store C, and
+// CT through a per-warp transpose buffer, while the next tile accumulates.
+// A symmetric product (A = X X^T and c A A^T + b A in Newton-Schulz) computes
+// only the tiles on or above the diagonal and writes each element twice, so
+// its result is exactly symmetric.  Every wait on an mbarrier gives up after
+// about a second and flags the error word instead.
 //
 // Any other case (fp32 storage, or leading dimensions that TMA cannot
 // address): a tiled CUDA-core kernel with fp32 arithmetic.
@@ -32,22 +35,8 @@ namespace gefen {
 
 namespace {
 
-constexpr int kBM = 128, kBN = 256, kBK = 64, kStages = 4;
-constexpr int kGemmThreads = 128;
-constexpr uint32_t kTileA = kBM * kBK * 2, kTileB = kBN * kBK * 2;  // bytes
-constexpr uint32_t kTmemCols = 256;
+constexpr int kBM = 128, kBK = 64;
 constexpr long long kSpin = 1ll << 31;
-
-struct alignas(1024) GemmSmem {
-    unsigned char a[kStages][kTileA];  // each 1024-byte aligned (swizzle atoms)
-    unsigned char b[kStages][kTileB];
-    unsigned long long full[kStages], empty[kStages], done;
-    uint32_t tmem;
-    int abort;
-    int consumed;  // k-tiles the MMA issuer took from the ring
-};
-// The transposed epilogue stages a 256 x 128 bf16 tile over the operand ring.
-static_assert(sizeof(GemmSmem::a) + sizeof(GemmSmem::b) >= kBN * kBM * 2, "staging fits the ring");
 
 __device__ __forceinline__ uint32_t saddr(const void* p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -94,19 +83,6 @@ __device__ __forceinline__ uint64_t desc_sw128(uint32_t addr) {
     d |= static_cast<uint64_t>(2) << 61;            // 128-byte swizzle
     return d;
 }
-// Instruction descriptor of kind::f16: fp32 accumulator (bits 4-5 = 1), bf16
-// A and B (bits 7-9, 10-12 = 1), both K-major, N / 8 at bit 17, M / 16 at 24.
-constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(kBN >> 3) << 17) |
-                            (static_cast<uint32_t>(kBM >> 4) << 24);
-
-__device__ __forceinline__ void umma_bf16(uint32_t tmem, uint64_t da, uint64_t db, uint32_t accumulate) {
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem),
-        "l"(da), "l"(db), "r"(kIdesc), "r"(accumulate)
-        : "memory");
-}
 __device__ __forceinline__ void umma_commit(uint32_t bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
                  : "memory");
@@ -140,24 +116,90 @@ struct GemmArgs {
     int ldc;
     __nv_bfloat16* CT;
     int ldct;
+    int sym;  // C is symmetric (M == N): only tiles on or above the diagonal are computed, each written twice
     int* err;
 };
 
-__global__ void __launch_bounds__(kGemmThreads, 1)
+// Per tile width BN: ring depth, bytes per stage, tensor-memory columns (two
+// accumulators, so the epilogue of one tile overlaps the next tile's MMAs).
+template <int BN>
+struct TcCfg {
+    static constexpr int kStagesN = BN == 256 ? 4 : 6;
+    static constexpr uint32_t kTileAB = kBM * kBK * 2, kTileBB = BN * kBK * 2;
+    static constexpr uint32_t kCols = 2 * BN;
+    // kind::f16 instruction descriptor: fp32 accumulator, bf16 A and B, both
+    // K-major, N / 8 at bit 17, M / 16 at bit 24
+    static constexpr uint32_t kIdescN = (1u << 4) | (1u << 7) | (1u << 10) |
+                                        (static_cast<uint32_t>(BN >> 3) << 17) |
+                                        (static_cast<uint32_t>(kBM >> 4) << 24);
+};
+
+template <int BN>
+struct alignas(1024) TcSmem {
+    using C = TcCfg<BN>;
+    unsigned char a[C::kStagesN][C::kTileAB];  // 1024-byte aligned tiles (swizzle atoms)
+    unsigned char b[C::kStagesN][C::kTileBB];
+    __nv_bfloat16 tr[4][32][40];  // per epilogue warp: 32 columns x 32 rows, padded rows
+    unsigned long long full[C::kStagesN], empty[C::kStagesN], acc_full[2], acc_empty[2];
+    uint32_t tmem;
+    int abort;
+    int consumed;  // k-tiles the MMA issuer took from the ring
+};
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void umma_bf16_n(uint32_t tmem, uint64_t da, uint64_t db, uint32_t idesc,
+                                            uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem),
+        "l"(da), "l"(db), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+// Tile t of the CTA's schedule: (m block, n block).  Symmetric products take
+// the tiles with m block <= n block only (BN == BM), n block by n block.
+__device__ __forceinline__ void tile_of(int t, int ntm, bool sym, int& mb, int& nb) {
+    if (!sym) {
+        mb = t % ntm;
+        nb = t / ntm;
+        return;
+    }
+    int j = static_cast<int>((sqrtf(8.0f * static_cast<float>(t) + 1.0f) - 1.0f) * 0.5f);
+    while (j * (j + 1) / 2 > t) --j;
+    while ((j + 1) * (j + 2) / 2 <= t) ++j;
+    nb = j;
+    mb = t - j * (j + 1) / 2;
+}
+
+constexpr int kTcThreads = 192;  // warp 0: TMA, warp 1: MMA, warps 2-5: epilogue
+
+// Persistent tcgen05 GEMM: each CTA takes tiles blockIdx.x, + gridDim.x, ...
+template <int BN>
+__global__ void __launch_bounds__(kTcThreads, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB, const GemmArgs G) {
+    using Cf = TcCfg<BN>;
+    constexpr int S = Cf::kStagesN;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     // aligned to 1024 bytes here: the launch asks for 1024 bytes of slack
-    GemmSmem& sm = *reinterpret_cast<GemmSmem*>(smem_raw + ((1024 - (saddr(smem_raw) & 1023)) & 1023));
+    TcSmem<BN>& sm = *reinterpret_cast<TcSmem<BN>*>(smem_raw + ((1024 - (saddr(smem_raw) & 1023)) & 1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int m0 = blockIdx.y * kBM, n0 = blockIdx.x * kBN;
     const int KT = (G.K + kBK - 1) / kBK;
+    const int ntm = (G.M + kBM - 1) / kBM, ntn = (G.N + BN - 1) / BN;
+    const bool sym = G.sym != 0;
+    const int ntiles = sym ? ntn * (ntn + 1) / 2 : ntm * ntn;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kStages; ++s) {
+        for (int s = 0; s < S; ++s) {
             mbar_init(saddr(&sm.full[s]), 1);
             mbar_init(saddr(&sm.empty[s]), 1);
         }
-        mbar_init(saddr(&sm.done), 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(saddr(&sm.acc_full[b]), 1);
+            mbar_init(saddr(&sm.acc_empty[b]), 4);  // one arrival per epilogue warp
+        }
         sm.abort = 0;
         sm.consumed = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -166,7 +208,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     }
     if (warp == 0) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(saddr(&sm.tmem)),
-                     "r"(kTmemCols)
+                     "r"(Cf::kCols)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
@@ -174,110 +216,170 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = sm.tmem;
+    volatile int* abort = &sm.abort;
 
     int issued = 0;  // thread 0: k-tiles whose loads were started
     if (threadIdx.x == 0) {
-        // producer: TMA loads of A and B k-tiles into the ring
-        for (int kt = 0; kt < KT; ++kt) {
-            const int s = kt % kStages;
-            if (kt >= kStages && !mbar_wait(saddr(&sm.empty[s]), static_cast<uint32_t>((kt / kStages - 1) & 1))) {
-                atomicExch(&sm.abort, 1);
-                break;
+        // producer: the A and B k-tiles of every tile of this CTA, in order
+        int ring = 0;
+        for (int t = blockIdx.x; t < ntiles && !*abort; t += gridDim.x) {
+            int mb, nb;
+            tile_of(t, ntm, sym, mb, nb);
+            for (int kt = 0; kt < KT; ++kt, ++ring) {
+                const int s = ring % S;
+                if (ring >= S && !mbar_wait(saddr(&sm.empty[s]), static_cast<uint32_t>((ring / S - 1) & 1))) {
+                    atomicExch(&sm.abort, 1);
+                    break;
+                }
+                const uint32_t bar = saddr(&sm.full[s]);
+                mbar_expect_tx(bar, Cf::kTileAB + Cf::kTileBB);
+                tma_load_2d(saddr(sm.a[s]), &mapA, kt * kBK, mb * kBM, bar);
+                tma_load_2d(saddr(sm.b[s]), &mapB, kt * kBK, nb * BN, bar);
+                issued = ring + 1;
             }
-            if (*static_cast<volatile int*>(&sm.abort)) break;
-            const uint32_t bar = saddr(&sm.full[s]);
-            mbar_expect_tx(bar, kTileA + kTileB);
-            tma_load_2d(saddr(sm.a[s]), &mapA, kt * kBK, m0, bar);
-            tma_load_2d(saddr(sm.b[s]), &mapB, kt * kBK, n0, bar);
-            issued = kt + 1;
         }
     } else if (threadIdx.x == 32) {
-        // MMA issuer: four K = 16 steps per stage, the stage freed by commit
-        int kt = 0;
-        for (; kt < KT; ++kt) {
-            const int s = kt % kStages;
-            if (!mbar_wait(saddr(&sm.full[s]), static_cast<uint32_t>((kt / kStages) & 1))) {
+        // MMA issuer: accumulator b = i & 1 for the CTA's i-th tile, reused
+        // once the epilogue has drained it
+        int ring = 0, i = 0;
+        for (int t = blockIdx.x; t < ntiles && !*abort; t += gridDim.x, ++i) {
+            const int b = i & 1;
+            if (i >= 2 && !mbar_wait(saddr(&sm.acc_empty[b]), static_cast<uint32_t>(((i >> 1) - 1) & 1))) {
                 atomicExch(&sm.abort, 1);
                 break;
             }
             tc_fence_after();
-            const uint32_t a0 = saddr(sm.a[s]), b0 = saddr(sm.b[s]);
-#pragma unroll
-            for (int kk = 0; kk < kBK / 16; ++kk)
-                umma_bf16(tmem, desc_sw128(a0 + kk * 32), desc_sw128(b0 + kk * 32), (kt | kk) != 0 ? 1u : 0u);
-            umma_commit(saddr(&sm.empty[s]));
-        }
-        sm.consumed = kt;
-        umma_commit(saddr(&sm.done));  // arrives once every MMA issued above has completed
-    }
-    __syncwarp();
-
-    // epilogue: warp w holds accumulator rows 32 w .. 32 w + 31 (TMEM lanes)
-    const bool ok = mbar_wait(saddr(&sm.done), 0u);
-    tc_fence_after();
-    // one decision for the whole CTA (the transposed store has a barrier)
-    if (!__syncthreads_and(ok && *static_cast<volatile int*>(&sm.abort) == 0)) {
-        if (threadIdx.x == 0) atomicExch(G.err, 1);
-    } else {
-        const int r = 32 * warp + lane, row = m0 + r;
-        __nv_bfloat16* stage = reinterpret_cast<__nv_bfloat16*>(sm.a[0]);  // CT staging: [col][row], 256 x 128
-        for (int c0 = 0; c0 < kBN; c0 += 32) {
-            float v[32];
-            tmem_ld32(tmem + (static_cast<uint32_t>(32 * warp) << 16) + static_cast<uint32_t>(c0), v);
-            if (row < G.M) {
-                if (G.beta != 0.0f && G.D != nullptr) {
-                    const __nv_bfloat16* d = G.D + static_cast<int64_t>(row) * G.ldd + n0 + c0;
-#pragma unroll
-                    for (int i = 0; i < 32; ++i)
-                        v[i] = G.alpha * v[i] + (n0 + c0 + i < G.N ? G.beta * __bfloat162float(d[i]) : 0.0f);
-                } else {
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) v[i] *= G.alpha;
+            const uint32_t acc = tmem + static_cast<uint32_t>(b * BN);
+            bool ok = true;
+            for (int kt = 0; kt < KT; ++kt, ++ring) {
+                const int s = ring % S;
+                if (!mbar_wait(saddr(&sm.full[s]), static_cast<uint32_t>((ring / S) & 1))) {
+                    atomicExch(&sm.abort, 1);
+                    ok = false;
+                    break;
                 }
-                if (G.C != nullptr) {
-                    __nv_bfloat16* c = G.C + static_cast<int64_t>(row) * G.ldc + n0 + c0;
-                    if (n0 + c0 + 32 <= G.N && ((reinterpret_cast<uintptr_t>(c) & 15u) == 0)) {
+                tc_fence_after();
+                const uint32_t a0 = saddr(sm.a[s]), b0 = saddr(sm.b[s]);
 #pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            __nv_bfloat162 h[4];
+                for (int kk = 0; kk < kBK / 16; ++kk)
+                    umma_bf16_n(acc, desc_sw128(a0 + kk * 32), desc_sw128(b0 + kk * 32), Cf::kIdescN,
+                                (kt | kk) != 0 ? 1u : 0u);
+                umma_commit(saddr(&sm.empty[s]));
+            }
+            umma_commit(saddr(&sm.acc_full[b]));  // arrives once this tile's MMAs have completed
+            if (!ok) break;
+        }
+        sm.consumed = ring;
+    } else if (warp >= 2) {
+        // epilogue: this warp reads accumulator rows 32 q .. 32 q + 31 (the
+        // TMEM lanes of warp id % 4)
+        const int q = warp & 3, e = warp - 2;
+        const int r = 32 * q + lane;
+        __nv_bfloat16(*tr)[40] = sm.tr[e];
+        int i = 0;
+        for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++i) {
+            const int b = i & 1;
+            const bool ok = mbar_wait(saddr(&sm.acc_full[b]), static_cast<uint32_t>((i >> 1) & 1));
+            tc_fence_after();
+            if (!__all_sync(0xffffffffu, ok) || *abort) {
+                atomicExch(&sm.abort, 1);
+                break;
+            }
+            int mb, nb;
+            tile_of(t, ntm, sym, mb, nb);
+            const int m0 = mb * kBM, n0 = nb * BN, row = m0 + r;
+            const bool diag = sym && mb * kBM + kBM > nb * BN;  // the tile holds elements below the diagonal
+            __nv_bfloat16* CT = sym ? G.C : G.CT;
+            const int ldct = sym ? G.ldc : G.ldct;
+            for (int c0 = 0; c0 < BN; c0 += 32) {
+                float v[32];
+                tmem_ld32(tmem + static_cast<uint32_t>(b * BN + c0) + (static_cast<uint32_t>(32 * q) << 16), v);
+                const int col0 = n0 + c0;
+                if (row < G.M) {
+                    if (G.beta != 0.0f && G.D != nullptr) {
+                        const __nv_bfloat16* d = G.D + static_cast<int64_t>(row) * G.ldd + col0;
+                        if (col0 + 32 <= G.N && (reinterpret_cast<uintptr_t>(d) & 15u) == 0) {
 #pragma unroll
-                            for (int i = 0; i < 4; ++i) h[i] = __floats2bfloat162_rn(v[8 * q + 2 * i], v[8 * q + 2 * i + 1]);
-                            *reinterpret_cast<uint4*>(c + 8 * q) = *reinterpret_cast<uint4*>(h);
+                            for (int qq = 0; qq < 4; ++qq) {
+                                const uint4 w = *reinterpret_cast<const uint4*>(d + 8 * qq);
+                                const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&w);
+#pragma unroll
+                                for (int k2 = 0; k2 < 4; ++k2) {
+                                    const float2 f = __bfloat1622float2(h[k2]);
+                                    v[8 * qq + 2 * k2] = G.alpha * v[8 * qq + 2 * k2] + G.beta * f.x;
+                                    v[8 * qq + 2 * k2 + 1] = G.alpha * v[8 * qq + 2 * k2 + 1] + G.beta * f.y;
+                                }
+                            }
+                        } else {
+#pragma unroll
+                            for (int k = 0; k < 32; ++k)
+                                v[k] = G.alpha * v[k] + (col0 + k < G.N ? G.beta * __bfloat162float(d[k]) : 0.0f);
                         }
                     } else {
-                        for (int i = 0; i < 32 && n0 + c0 + i < G.N; ++i) c[i] = __float2bfloat16_rn(v[i]);
+#pragma unroll
+                        for (int k = 0; k < 32; ++k) v[k] *= G.alpha;
+                    }
+                    if (G.C != nullptr) {
+                        __nv_bfloat16* c = G.C + static_cast<int64_t>(row) * G.ldc + col0;
+                        if (!diag && col0 + 32 <= G.N && (reinterpret_cast<uintptr_t>(c) & 15u) == 0) {
+#pragma unroll
+                            for (int qq = 0; qq < 4; ++qq) {
+                                __nv_bfloat162 h[4];
+#pragma unroll
+                                for (int k2 = 0; k2 < 4; ++k2)
+                                    h[k2] = __floats2bfloat162_rn(v[8 * qq + 2 * k2], v[8 * qq + 2 * k2 + 1]);
+                                *reinterpret_cast<uint4*>(c + 8 * qq) = *reinterpret_cast<uint4*>(h);
+                            }
+                        } else {
+#pragma unroll
+                            for (int k = 0; k < 32; ++k)
+                                if (col0 + k < G.N && (!sym || row <= col0 + k)) c[k] = __float2bfloat16_rn(v[k]);
+                        }
                     }
                 }
-            }
-            if (G.CT != nullptr) {
+                if (CT != nullptr) {
+                    // transpose through this warp's buffer: lane l then owns
+                    // column col0 + l, rows m0 + 32 q .. + 31
 #pragma unroll
-                for (int i = 0; i < 32; ++i) stage[(c0 + i) * kBM + r] = __float2bfloat16_rn(v[i]);
+                    for (int k = 0; k < 32; ++k) tr[k][lane] = __float2bfloat16_rn(v[k]);
+                    __syncwarp();
+                    const int jcol = col0 + lane, i0 = m0 + 32 * q;
+                    if (jcol < G.N) {
+                        __nv_bfloat16* ct = CT + static_cast<int64_t>(jcol) * ldct + i0;
+                        if (!diag && i0 + 32 <= G.M && (reinterpret_cast<uintptr_t>(ct) & 15u) == 0) {
+#pragma unroll
+                            for (int qq = 0; qq < 4; ++qq)
+                                *reinterpret_cast<uint4*>(ct + 8 * qq) = *reinterpret_cast<const uint4*>(&tr[lane][8 * qq]);
+                        } else {
+                            for (int k = 0; k < 32; ++k)
+                                if (i0 + k < G.M && (!sym || i0 + k < jcol)) ct[k] = tr[lane][k];
+                        }
+                    }
+                    __syncwarp();
+                }
             }
-        }
-        if (G.CT != nullptr) {
-            __syncthreads();
-            // rows of CT: column n0 + j of C, elements m0 .. m0 + 127 (256 bytes)
-            for (int j = warp; j < kBN; j += kGemmThreads / 32) {
-                const int col = n0 + j;
-                if (col >= G.N) break;
-                __nv_bfloat16* ct = G.CT + static_cast<int64_t>(col) * G.ldct + m0;
-                const __nv_bfloat16* src = stage + j * kBM;
-                for (int i = lane; i < kBM; i += 32)
-                    if (m0 + i < G.M) ct[i] = src[i];
-            }
+            // this accumulator is drained: the MMA issuer may reuse it
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(saddr(&sm.acc_empty[b]));
         }
     }
+    __syncwarp();
     tc_fence_before();
     __syncthreads();
-    if (threadIdx.x == 0 && sm.consumed < issued) {
-        // an aborted pipeline: wait (bounded) for the loads still in flight
-        for (int kt = sm.consumed; kt < issued; ++kt)
-            mbar_wait(saddr(&sm.full[kt % kStages]), static_cast<uint32_t>((kt / kStages) & 1));
+    if (*abort) {
+        if (threadIdx.x == 0) {
+            atomicExch(G.err, 1);
+            // wait (bounded) for the loads still in flight
+            for (int k = sm.consumed; k < issued; ++k)
+                mbar_wait(saddr(&sm.full[k % S]), static_cast<uint32_t>((k / S) & 1));
+        }
     }
     if (warp == 0) {
         __syncwarp();
         tc_fence_after();
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(Cf::kCols)
+                     : "memory");
     }
 }
 
@@ -381,13 +483,30 @@ bool gemm_tc_usable(int lda, int ldb, const void* A, const void* B) {
            (reinterpret_cast<uintptr_t>(B) & 15u) == 0 && encode_fn() != nullptr;
 }
 
+template <int BN>
+cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const GemmArgs& G, cudaStream_t st) {
+    const int smem = static_cast<int>(sizeof(TcSmem<BN>)) + 1024;
+    cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    const int ntm = (G.M + kBM - 1) / kBM, ntn = (G.N + BN - 1) / BN;
+    const int ntiles = G.sym ? ntn * (ntn + 1) / 2 : ntm * ntn;
+    const int grid = std::min(ntiles, device_sm_count());
+    k_gemm_tc<BN><<<grid, kTcThreads, smem, st>>>(ma, mb, G);
+    return cudaGetLastError();
+}
+
 cudaError_t gemm_bf16_nt(int M, int N, int K, float alpha, const void* A, int lda, const void* B, int ldb,
                          float beta, const void* D, int ldd, void* C, int ldc, void* CT, int ldct, int* err,
-                         cudaStream_t st) {
+                         cudaStream_t st, bool sym) {
     if (M <= 0 || N <= 0) return cudaSuccess;
+    if (sym && (M != N || CT != nullptr || C == nullptr)) return cudaErrorInvalidValue;
     if (K > 0 && gemm_tc_usable(lda, ldb, A, B)) {
+        // 256-wide tiles when there are enough of them for every SM, else
+        // (and for symmetric products) 128-wide ones
+        const int64_t tiles256 = static_cast<int64_t>((M + kBM - 1) / kBM) * ((N + 255) / 256);
+        const int bn = (sym || tiles256 < device_sm_count()) ? 128 : 256;
         CUtensorMap ma, mb;
-        if (!make_map(&ma, A, M, K, lda, kBM) || !make_map(&mb, B, N, K, ldb, kBN)) return cudaErrorInvalidValue;
+        if (!make_map(&ma, A, M, K, lda, kBM) || !make_map(&mb, B, N, K, ldb, bn)) return cudaErrorInvalidValue;
         GemmArgs G;
         G.M = M;
         G.N = N;
@@ -400,13 +519,9 @@ cudaError_t gemm_bf16_nt(int M, int N, int K, float alpha, const void* A, int ld
         G.ldc = ldc;
         G.CT = static_cast<__nv_bfloat16*>(CT);
         G.ldct = ldct;
+        G.sym = sym ? 1 : 0;
         G.err = err;
-        const int smem = static_cast<int>(sizeof(GemmSmem)) + 1024;
-        cudaError_t e = cudaFuncSetAttribute(k_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-        if (e != cudaSuccess) return e;
-        const dim3 grid((N + kBN - 1) / kBN, (M + kBM - 1) / kBM);
-        k_gemm_tc<<<grid, kGemmThreads, smem, st>>>(ma, mb, G);
-        return cudaGetLastError();
+        return bn == 128 ? launch_tc<128>(ma, mb, G, st) : launch_tc<256>(ma, mb, G, st);
     }
     const dim3 grid((N + 63) / 64, (M + 63) / 64);
     k_gemm_simt<__nv_bfloat16><<<grid, 256, 0, st>>>(
@@ -441,7 +556,7 @@ extern "C" gefen_status_t gefen_gemm_bf16(int32_t M, int32_t N, int32_t K, float
     if (gefen_status_t s = check_device(); s != GEFEN_OK) return s;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     int* err = static_cast<int*>(workspace);
-    if (gemm_bf16_nt(M, N, K, alpha, A, lda, B, ldb, beta, D, ldd, C, ldc, CT, ldct, err, st) != cudaSuccess)
+    if (gemm_bf16_nt(M, N, K, alpha, A, lda, B, ldb, beta, D, ldd, C, ldc, CT, ldct, err, st, false) != cudaSuccess)
         return GEFEN_ECUDA;
     return GEFEN_OK;
 }

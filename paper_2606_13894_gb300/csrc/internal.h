@@ -31,9 +31,11 @@ cudaError_t prepare_histogram();
 // written as C and/or as its transpose CT (N x M); bf16 storage with fp32
 // accumulation (tcgen05 when TMA can address A and B), or fp32 throughout.
 // D, C, CT nullable.  err: device word set when a bounded wait gave up.
+// sym: the result is symmetric (M == N, C given, CT not): on the tensor cores
+// only the tiles on or above the diagonal are computed and mirrored.
 cudaError_t gemm_bf16_nt(int M, int N, int K, float alpha, const void* A, int lda, const void* B, int ldb,
                          float beta, const void* D, int ldd, void* C, int ldc, void* CT, int ldct, int* err,
-                         cudaStream_t st);
+                         cudaStream_t st, bool sym = false);
 cudaError_t gemm_f32_nt(int M, int N, int K, float alpha, const float* A, int lda, const float* B, int ldb,
                         float beta, const float* D, int ldd, float* C, int ldc, float* CT, int ldct,
                         cudaStream_t st);

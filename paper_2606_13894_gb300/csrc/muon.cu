@@ -40,7 +40,7 @@ struct MuonLayout {
     size_t hdr, snew, part, p0, p1, q0, q1, ga, gb, total;
 };
 
-// header (256 B; word 0: a bounded wait gave up) | new scales | norm
+// header (256 B; word 0: a bounded wait gave up; byte 16: 1 / ||U||) | new scales | norm
 // partials | two rows x cols buffers (U's layout) | two cols x rows buffers
 // (transposed) | A | B
 MuonLayout muon_layout(int64_t rows, int64_t cols, int64_t period, bool bf16) {
@@ -111,6 +111,187 @@ __global__ void __launch_bounds__(kMuThreads) k_muon_absmax(MuonArgs A) {
     }
 }
 
+// Vector forms (period % 8 == 0, n % 8 == 0, codes 8-byte aligned): a thread
+// takes eight consecutive elements -- one 16-byte load of g, one 8-byte load
+// of codes, all in one block -- with the same arithmetic per element as the
+// scalar forms.
+__device__ __forceinline__ void load8(const MuonArgs& A, int64_t v, float (&g)[8], uint32_t (&c)[8]) {
+    const uint4 gw = reinterpret_cast<const uint4*>(A.grads)[v];
+    const uint2 cw = reinterpret_cast<const uint2*>(A.codes)[v];
+    const uint32_t gg[4] = {gw.x, gw.y, gw.z, gw.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        g[2 * i] = bf16_lo(gg[i]);
+        g[2 * i + 1] = bf16_hi(gg[i]);
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        c[i] = (cw.x >> (8 * i)) & 0xFFu;
+        c[4 + i] = (cw.y >> (8 * i)) & 0xFFu;
+    }
+}
+
+__global__ void __launch_bounds__(kMuThreads) k_muon_absmax8(MuonArgs A) {
+    __shared__ float s_dec[kMaxLevels];
+    if (threadIdx.x < kMaxLevels) s_dec[threadIdx.x] = threadIdx.x < A.k ? A.cb_dec[threadIdx.x] : 0.0f;
+    __syncthreads();
+    const int64_t nv = A.n >> 3;
+    for (int64_t v = blockIdx.x * static_cast<int64_t>(kMuThreads) + threadIdx.x; v < nv;
+         v += static_cast<int64_t>(gridDim.x) * kMuThreads) {
+        const int64_t bi = muon_block(A, v << 3);
+        float g[8];
+        uint32_t c[8];
+        load8(A, v, g, c);
+        const float mus = A.mu * A.scale[bi];
+        float am = 0.0f;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) am = fmaxf(am, fabsf(fmaf(A.omm, g[i], mus * s_dec[c[i]])));
+        unsigned* dst = reinterpret_cast<unsigned int*>(A.snew) + bi;
+        const unsigned live = __activemask();
+        const int first = __ffs(live) - 1;
+        const long long b0 = __shfl_sync(live, static_cast<long long>(bi), first);
+        const unsigned ab = __float_as_uint(am);
+        if (__all_sync(live, bi == b0)) {
+            const unsigned wm = __reduce_max_sync(live, ab);
+            if ((threadIdx.x & 31) == first) atomicMax(dst, wm);
+        } else {
+            atomicMax(dst, ab);
+        }
+    }
+}
+
+template <bool BF16>
+__global__ void __launch_bounds__(kMuThreads) k_muon_encode8(MuonArgs A) {
+    __shared__ float s_dec[kMaxLevels], s_mid[kMaxLevels];
+    __shared__ double s_red[kMuThreads / 32];
+    const int t = threadIdx.x;
+    if (t < kMaxLevels) {
+        s_dec[t] = t < A.k ? A.cb_dec[t] : 0.0f;
+        s_mid[t] = (t < A.k - 1) ? 0.5f * (A.cb_enc[t] + A.cb_enc[t + 1]) : INFINITY;
+    }
+    __syncthreads();
+    const int zero_code = level_search(s_mid, 0.0f);
+    double acc = 0.0;
+    const int64_t nv = A.n >> 3;
+    for (int64_t v = blockIdx.x * static_cast<int64_t>(kMuThreads) + t; v < nv;
+         v += static_cast<int64_t>(gridDim.x) * kMuThreads) {
+        const int64_t bi = muon_block(A, v << 3);
+        float g[8];
+        uint32_t c[8];
+        load8(A, v, g, c);
+        const float mus = A.mu * A.scale[bi];
+        const float sn = A.snew[bi];
+        float u[8];
+        uint32_t cw[2] = {0u, 0u};
+        float sq = 0.0f;  // squares of the stored update, exact in fp32 for bf16 values
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            const float m = fmaf(A.omm, g[i], mus * s_dec[c[i]]);
+            const uint32_t code = sn > 0.0f ? static_cast<uint32_t>(level_search(s_mid, __fdiv_rn(m, sn)))
+                                            : static_cast<uint32_t>(zero_code);
+            cw[i >> 2] |= code << (8 * (i & 3));
+            u[i] = A.nesterov ? fmaf(A.mu, m - g[i], g[i]) : m;
+            if (BF16) u[i] = __bfloat162float(__float2bfloat16_rn(u[i]));
+        }
+        reinterpret_cast<uint2*>(A.codes)[v] = make_uint2(cw[0], cw[1]);
+        if (BF16) {
+            __nv_bfloat162 h[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) h[i] = __floats2bfloat162_rn(u[2 * i], u[2 * i + 1]);
+            reinterpret_cast<uint4*>(A.u)[v] = *reinterpret_cast<uint4*>(h);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) sq = fmaf(u[i], u[i], sq);
+            acc += static_cast<double>(sq);
+        } else {
+            float4* uo = reinterpret_cast<float4*>(A.u) + 2 * v;
+            uo[0] = make_float4(u[0], u[1], u[2], u[3]);
+            uo[1] = make_float4(u[4], u[5], u[6], u[7]);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) acc += static_cast<double>(u[i]) * u[i];
+        }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if ((t & 31) == 0) s_red[t >> 5] = acc;
+    __syncthreads();
+    if (t == 0) {
+        double sum = 0.0;
+        for (int w = 0; w < kMuThreads / 32; ++w) sum += s_red[w];
+        A.part[blockIdx.x] = sum;
+    }
+}
+
+// 1 / max(||U||, eps) from the partials, summed in one fixed order.
+__global__ void __launch_bounds__(kMuThreads) k_muon_inv(const double* __restrict__ part, int nparts, double eps,
+                                                        float* __restrict__ inv_out) {
+    __shared__ double s_sum[kMuThreads];
+    double ps = 0.0;
+    for (int i = threadIdx.x; i < nparts; i += kMuThreads) ps += part[i];
+    s_sum[threadIdx.x] = ps;
+    __syncthreads();
+    for (int w = kMuThreads / 2; w > 0; w >>= 1) {
+        if (threadIdx.x < w) s_sum[threadIdx.x] += s_sum[threadIdx.x + w];
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) *inv_out = static_cast<float>(1.0 / fmax(sqrt(s_sum[0]), eps));
+}
+
+// X = U / ||U|| in place (rows x cols) and, when ut is given, its transpose
+// (cols x rows), 32 x 32 tiles through shared memory; the new scales are
+// committed on the way.
+template <typename T>
+__global__ void __launch_bounds__(256) k_muon_scale_t(T* __restrict__ u, T* __restrict__ ut, int rows, int cols,
+                                                     const float* __restrict__ inv_p, float* __restrict__ scale,
+                                                     const float* __restrict__ snew, int64_t nb) {
+    __shared__ T tile[32][33];
+    const float inv = *inv_p;
+    const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
+    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+    for (int i = ty; i < 32; i += 8) {
+        if (r0 + i < rows && c0 + tx < cols) {
+            T* p = u + static_cast<int64_t>(r0 + i) * cols + c0 + tx;
+            T y;
+            if constexpr (sizeof(T) == 2) y = __float2bfloat16_rn(__bfloat162float(*p) * inv);
+            else y = *p * inv;
+            *p = y;
+            tile[i][tx] = y;
+        }
+    }
+    const int64_t cta = static_cast<int64_t>(blockIdx.y) * gridDim.x + blockIdx.x;
+    const int64_t ncta = static_cast<int64_t>(gridDim.x) * gridDim.y;
+    for (int64_t b = cta * 256 + threadIdx.x; b < nb; b += ncta * 256) scale[b] = snew[b];
+    if (ut == nullptr) return;
+    __syncthreads();
+    for (int i = ty; i < 32; i += 8)
+        if (c0 + i < cols && r0 + tx < rows) ut[static_cast<int64_t>(c0 + i) * rows + r0 + tx] = tile[tx][i];
+}
+
+// theta = theta * decay - step * X, four elements per thread.
+template <bool BF16>
+__global__ void __launch_bounds__(kMuThreads) k_muon_update4(float* __restrict__ theta, const void* __restrict__ x,
+                                                          int64_t n4, float decay, float step) {
+    for (int64_t v = blockIdx.x * static_cast<int64_t>(kMuThreads) + threadIdx.x; v < n4;
+         v += static_cast<int64_t>(gridDim.x) * kMuThreads) {
+        float xv[4];
+        if (BF16) {
+            const uint2 w = reinterpret_cast<const uint2*>(x)[v];
+            xv[0] = bf16_lo(w.x);
+            xv[1] = bf16_hi(w.x);
+            xv[2] = bf16_lo(w.y);
+            xv[3] = bf16_hi(w.y);
+        } else {
+            const float4 f = reinterpret_cast<const float4*>(x)[v];
+            xv[0] = f.x; xv[1] = f.y; xv[2] = f.z; xv[3] = f.w;
+        }
+        float4 t4 = reinterpret_cast<float4*>(theta)[v];
+        t4.x = fmaf(-step, xv[0], decay * t4.x);
+        t4.y = fmaf(-step, xv[1], decay * t4.y);
+        t4.z = fmaf(-step, xv[2], decay * t4.z);
+        t4.w = fmaf(-step, xv[3], decay * t4.w);
+        reinterpret_cast<float4*>(theta)[v] = t4;
+    }
+}
+
 // Re-encode, write the update U and each CTA's partial sum of U^2.
 template <bool BF16>
 __global__ void __launch_bounds__(kMuThreads) k_muon_encode(MuonArgs A) {
@@ -153,38 +334,6 @@ __global__ void __launch_bounds__(kMuThreads) k_muon_encode(MuonArgs A) {
     }
 }
 
-// Normalise U and commit the new scales.  Every CTA sums the partials in the
-// same fixed order (thread t: partials t, t + 256, ...; then a fixed tree),
-// so all use the same norm.
-template <bool BF16>
-__global__ void __launch_bounds__(kMuThreads) k_muon_normalise(MuonArgs A, int nparts, double eps) {
-    __shared__ double s_sum[kMuThreads];
-    __shared__ float s_inv;
-    double ps = 0.0;
-    for (int i = threadIdx.x; i < nparts; i += kMuThreads) ps += A.part[i];
-    s_sum[threadIdx.x] = ps;
-    __syncthreads();
-    for (int w = kMuThreads / 2; w > 0; w >>= 1) {
-        if (threadIdx.x < w) s_sum[threadIdx.x] += s_sum[threadIdx.x + w];
-        __syncthreads();
-    }
-    if (threadIdx.x == 0) s_inv = static_cast<float>(1.0 / fmax(sqrt(s_sum[0]), eps));
-    __syncthreads();
-    const float inv = s_inv;
-    const int64_t nb = A.n / A.period;
-    for (int64_t e = blockIdx.x * static_cast<int64_t>(kMuThreads) + threadIdx.x; e < A.n;
-         e += static_cast<int64_t>(gridDim.x) * kMuThreads) {
-        if (BF16) {
-            __nv_bfloat16* u = reinterpret_cast<__nv_bfloat16*>(A.u);
-            u[e] = __float2bfloat16_rn(__bfloat162float(u[e]) * inv);
-        } else {
-            float* u = reinterpret_cast<float*>(A.u);
-            u[e] *= inv;
-        }
-        if (e < nb) A.scale[e] = A.snew[e];
-    }
-}
-
 template <bool BF16>
 __global__ void __launch_bounds__(kMuThreads) k_muon_update(float* __restrict__ theta, const void* __restrict__ x,
                                                          int64_t n, float decay, float step) {
@@ -194,19 +343,6 @@ __global__ void __launch_bounds__(kMuThreads) k_muon_update(float* __restrict__ 
                               : reinterpret_cast<const float*>(x)[e];
         theta[e] = fmaf(-step, xv, decay * theta[e]);
     }
-}
-
-// out (cols x rows) = in (rows x cols)^T, 32 x 32 tiles through shared memory.
-template <typename T>
-__global__ void __launch_bounds__(256) k_transpose(const T* __restrict__ in, T* __restrict__ out, int rows, int cols) {
-    __shared__ T tile[32][33];
-    const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
-    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
-    for (int i = ty; i < 32; i += 8)
-        if (r0 + i < rows && c0 + tx < cols) tile[i][tx] = in[static_cast<int64_t>(r0 + i) * cols + c0 + tx];
-    __syncthreads();
-    for (int i = ty; i < 32; i += 8)
-        if (c0 + i < cols && r0 + tx < rows) out[static_cast<int64_t>(c0 + i) * rows + r0 + tx] = tile[tx][i];
 }
 
 }  // namespace
@@ -269,17 +405,36 @@ extern "C" gefen_status_t gefen_muon_step(int64_t rows, int64_t cols, int64_t pe
     A.u = P0;
 
     const int grid = static_cast<int>(std::min<int64_t>(kMuPartials, (n + kMuThreads - 1) / kMuThreads));
+    // eight elements per thread when whole groups of eight share a block
+    const bool vec = period % 8 == 0 && n % 8 == 0 && (reinterpret_cast<uintptr_t>(codes) & 7u) == 0;
     if (cudaMemsetAsync(A.snew, 0, static_cast<size_t>(n / period) * sizeof(float), st) != cudaSuccess)
         return GEFEN_ECUDA;
-    k_muon_absmax<<<grid, kMuThreads, 0, st>>>(A);
+    if (vec) k_muon_absmax8<<<grid, kMuThreads, 0, st>>>(A);
+    else k_muon_absmax<<<grid, kMuThreads, 0, st>>>(A);
     if (bf16) {
-        k_muon_encode<true><<<grid, kMuThreads, 0, st>>>(A);
-        k_muon_normalise<true><<<grid, kMuThreads, 0, st>>>(A, grid, hp.eps);
+        if (vec) k_muon_encode8<true><<<grid, kMuThreads, 0, st>>>(A);
+        else k_muon_encode<true><<<grid, kMuThreads, 0, st>>>(A);
     } else {
-        k_muon_encode<false><<<grid, kMuThreads, 0, st>>>(A);
-        k_muon_normalise<false><<<grid, kMuThreads, 0, st>>>(A, grid, hp.eps);
+        if (vec) k_muon_encode8<false><<<grid, kMuThreads, 0, st>>>(A);
+        else k_muon_encode<false><<<grid, kMuThreads, 0, st>>>(A);
     }
+    float* inv = reinterpret_cast<float*>(ws + L.hdr + 16);
+    k_muon_inv<<<1, kMuThreads, 0, st>>>(A.part, grid, hp.eps, inv);
     if (cudaGetLastError() != cudaSuccess) return GEFEN_ECUDA;
+    // X = U / ||U|| in place, with its transpose when Newton-Schulz follows
+    {
+        const dim3 tg(static_cast<unsigned>((cols + 31) / 32), static_cast<unsigned>((rows + 31) / 32));
+        void* ut = hp.ns_steps > 0 ? Q0 : nullptr;
+        if (bf16)
+            k_muon_scale_t<__nv_bfloat16><<<tg, 256, 0, st>>>(static_cast<__nv_bfloat16*>(P0),
+                                                              static_cast<__nv_bfloat16*>(ut), static_cast<int>(rows),
+                                                              static_cast<int>(cols), inv, scale, A.snew, n / period);
+        else
+            k_muon_scale_t<float><<<tg, 256, 0, st>>>(static_cast<float*>(P0), static_cast<float*>(ut),
+                                                     static_cast<int>(rows), static_cast<int>(cols), inv, scale,
+                                                     A.snew, n / period);
+        if (cudaGetLastError() != cudaSuccess) return GEFEN_ECUDA;
+    }
 
     // Newton-Schulz on X (s x n) and T = X^T (n x s): the P buffers hold U's
     // layout (rows x cols), the Q buffers the transposed one
@@ -288,21 +443,13 @@ extern "C" gefen_status_t gefen_muon_step(int64_t rows, int64_t cols, int64_t pe
     const float a = static_cast<float>(hp.ns_a), b = static_cast<float>(hp.ns_b), c = static_cast<float>(hp.ns_c);
     void* U = P0;
     if (hp.ns_steps > 0) {
-        const dim3 tg(static_cast<unsigned>((cols + 31) / 32), static_cast<unsigned>((rows + 31) / 32));
-        if (bf16)
-            k_transpose<__nv_bfloat16><<<tg, 256, 0, st>>>(static_cast<const __nv_bfloat16*>(P0),
-                                                           static_cast<__nv_bfloat16*>(Q0), static_cast<int>(rows),
-                                                           static_cast<int>(cols));
-        else
-            k_transpose<float><<<tg, 256, 0, st>>>(static_cast<const float*>(P0), static_cast<float*>(Q0),
-                                                  static_cast<int>(rows), static_cast<int>(cols));
         void *X = wide ? P0 : Q0, *T = wide ? Q0 : P0, *Xn = wide ? P1 : Q1, *Tn = wide ? Q1 : P1;
         for (int it = 0; it < hp.ns_steps; ++it) {
             cudaError_t e;
             if (bf16) {
-                e = gemm_bf16_nt(s, s, nn, 1.0f, X, nn, X, nn, 0.0f, nullptr, 0, GA, s, nullptr, 0, err, st);
+                e = gemm_bf16_nt(s, s, nn, 1.0f, X, nn, X, nn, 0.0f, nullptr, 0, GA, s, nullptr, 0, err, st, true);
                 if (e == cudaSuccess)
-                    e = gemm_bf16_nt(s, s, s, c, GA, s, GA, s, b, GA, s, GB, s, nullptr, 0, err, st);
+                    e = gemm_bf16_nt(s, s, s, c, GA, s, GA, s, b, GA, s, GB, s, nullptr, 0, err, st, true);
                 if (e == cudaSuccess)
                     e = gemm_bf16_nt(s, nn, s, 1.0f, GB, s, T, s, a, X, nn, Xn, nn, Tn, s, err, st);
             } else {
@@ -322,10 +469,13 @@ extern "C" gefen_status_t gefen_muon_step(int64_t rows, int64_t cols, int64_t pe
     }
     const double adj = hp.lr * std::sqrt(std::max(1.0, static_cast<double>(rows) / static_cast<double>(cols)));
     const float decay = static_cast<float>(1.0 - hp.lr * hp.weight_decay);
-    if (bf16)
-        k_muon_update<true><<<grid, kMuThreads, 0, st>>>(params, U, n, decay, static_cast<float>(adj));
-    else
-        k_muon_update<false><<<grid, kMuThreads, 0, st>>>(params, U, n, decay, static_cast<float>(adj));
+    if (n % 4 == 0) {
+        if (bf16) k_muon_update4<true><<<grid, kMuThreads, 0, st>>>(params, U, n / 4, decay, static_cast<float>(adj));
+        else k_muon_update4<false><<<grid, kMuThreads, 0, st>>>(params, U, n / 4, decay, static_cast<float>(adj));
+    } else {
+        if (bf16) k_muon_update<true><<<grid, kMuThreads, 0, st>>>(params, U, n, decay, static_cast<float>(adj));
+        else k_muon_update<false><<<grid, kMuThreads, 0, st>>>(params, U, n, decay, static_cast<float>(adj));
+    }
     if (cudaGetLastError() != cudaSuccess) return GEFEN_ECUDA;
     return GEFEN_OK;
 }
