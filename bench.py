@@ -437,6 +437,7 @@ def run_gpu(args, world, rank, local):
     if world == 1 and not args.no_extras:
         res["gpt2_125m"] = gpt2_figures(G, synth, dev, args, stream, hbm)
         res["flat_sweep"] = flat_sweep(G, synth, dev, stream, hbm)
+        res["gefen_muon"] = muon_figures(G, dev)
     if rank == 0 and not args.no_cpu_baseline:
         res["cpu_baseline"] = cpu_baseline(args)
     return res
@@ -539,6 +540,51 @@ def refit_microbench(G, synth, dev, n=MICRO_N, bins=MICRO_BINS):
             "nonempty_cells": int((hist > 0).sum().item()),
             "hist_ms": hist_dp_ms - dp_ms, "dp_ms": dp_ms, "total_ms": hist_dp_ms,
             "hist_gbs": 4 * n / ((hist_dp_ms - dp_ms) * 1e-3) / 1e9}
+
+
+def muon_figures(G, dev, shapes=((2048, 8192), (8192, 2048), (2048, 2048)), warm=3, reps=5, steps_ns=5):
+    """Gefen-Muon (bf16 products on the tensor cores): CUDA-event time of one
+    gefen_muon_step per shape (period = cols, 5 Newton-Schulz steps) and the
+    Newton-Schulz flops over that whole step time, against the measured bf16
+    peak."""
+    out = {}
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            pk = json.load(f)
+        peak, kind = float(pk["bf16_tflops"]), "measured"
+    except Exception:
+        peak, kind = 1900.0, "fallback"
+    for rows, cols in shapes:
+        n = rows * cols
+        g = torch.Generator(device=dev).manual_seed(rows + cols)
+        th = torch.randn(n, device=dev, generator=g) * 0.02
+        gr = (torch.randn(n, device=dev, generator=g) * 1e-3).to(torch.bfloat16)
+        codes = torch.full((n,), 128, dtype=torch.uint8, device=dev)
+        sc = torch.zeros(n // cols, device=dev)
+        cb = torch.linspace(-1, 1, K, device=dev)
+        ws = None
+        for _ in range(warm):
+            ws = G.gefen_muon_step(rows, cols, cols, th, gr, codes, sc, cb, cb, lr=1e-3, ns_steps=steps_ns,
+                                   flags=G.GEFEN_MUON_BF16_GEMM, workspace_buf=ws)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            ws = G.gefen_muon_step(rows, cols, cols, th, gr, codes, sc, cb, cb, lr=1e-3, ns_steps=steps_ns,
+                                   flags=G.GEFEN_MUON_BF16_GEMM, workspace_buf=ws)
+        e1.record()
+        torch.cuda.synchronize()
+        G.gefen_step_status(ws)
+        ms = e0.elapsed_time(e1) / reps
+        sm, lg = min(rows, cols), max(rows, cols)
+        flops = steps_ns * (2 * 2 * sm * sm * lg + 2 * sm ** 3)  # X X^T, A A, B X per step
+        tf = flops / (ms * 1e-3) / 1e12
+        out[f"{rows}x{cols}"] = {"ms": ms, "ns_tflops": tf, "frac": tf / peak}
+        del th, gr, codes, sc, ws
+        torch.cuda.empty_cache()
+    return {"shapes": out, "peak_tflops": peak, "peak_kind": kind,
+            "note": "Newton-Schulz flops (2 s^2 n + 2 s^3 + 2 s^2 n per step) over the whole step time "
+                    "(element-wise kernels included), bf16 products with fp32 accumulation"}
 
 
 def run_e2e(G, cad, args, stream):
@@ -710,10 +756,18 @@ def main():
     ap.add_argument("--microbench-only", action="store_true",
                     help="run only the refit micro-benchmark and print its figures (one GPU)")
     ap.add_argument("--micro-values", type=int, default=MICRO_N, help="refit micro-benchmark values (multiple of 4096)")
+    ap.add_argument("--muon-only", default=None, metavar="ROWSxCOLS",
+                    help="time only gefen_muon_step (bf16 products) on one matrix shape and print its figures")
     ap.add_argument("--micro-bins", type=int, default=MICRO_BINS, help="refit micro-benchmark histogram cells")
     ap.add_argument("--workload", default=WORKLOAD,
                     help="llama-1.5b (default), gpt2-125m, tiny, or flat:N:P (one tensor, blocks of P)")
     args = ap.parse_args()
+    if args.muon_only:
+        from paper_2606_13894_gb300 import gefen as G
+        G.load()
+        r, c = (int(v) for v in args.muon_only.lower().split("x"))
+        print(json.dumps({"gefen_muon": muon_figures(G, torch.device("cuda", 0), shapes=((r, c),))}), flush=True)
+        return
     if args.microbench_only:
         from paper_2606_13894_gb300 import gefen as G
         from paper_2606_13894_gb300 import synth
