@@ -325,15 +325,27 @@ size_t gefen_muon_workspace_size(int64_t rows, int64_t cols, int64_t period, uin
  * leading dimensions lda >= K, ldb >= K, ldd >= N, ldc >= N; CT (nullable)
  * receives C transposed (N x M, ldct >= M); C may be NULL when CT is given; D
  * is read only when beta != 0.  fp32 accumulation; each output rounded once
- * to bf16.  With 16-byte aligned A and B and lda, ldb multiples of 8 the
- * product runs on the tensor cores (tcgen05, operands staged by TMA), else on
- * the CUDA cores.  workspace: >= 256 bytes, 256-byte aligned; its word 0 is
+ * to bf16.  When every matrix it touches (A, B, C, CT, and D if read) is
+ * 16-byte aligned with a leading dimension that is a multiple of 8, the
+ * product runs on the tensor cores (tcgen05; operands staged and results
+ * written by TMA), else on the CUDA cores.  workspace: >= 256 bytes, 256-byte aligned; its word 0 is
  * set if a bounded wait gave up (read it with gefen_step_status). */
 gefen_status_t gefen_gemm_bf16(int32_t M, int32_t N, int32_t K, float alpha, const uint16_t* A,
                                int32_t lda, const uint16_t* B, int32_t ldb, float beta,
                                const uint16_t* D, int32_t ldd, uint16_t* C, int32_t ldc,
                                uint16_t* CT, int32_t ldct, void* workspace, size_t workspace_bytes,
                                gefen_stream_t stream);
+/* The symmetric product of the same iteration (X X^T and its powers):
+ *   C = alpha * A * A^T + beta * D
+ * A: N x K, C and D: N x N, row-major bf16, lda >= K, ldc >= N, ldd >= N; D
+ * is read only when beta != 0 and must then be symmetric.  C is symmetric bit
+ * for bit: on the tensor cores (conditions as for gefen_gemm_bf16) only the
+ * tiles on or above the diagonal are computed and each is also written
+ * mirrored; on the CUDA cores C[i][j] and C[j][i] sum the same products in the
+ * same order.  C must not overlap A or D.  workspace as for gefen_gemm_bf16. */
+gefen_status_t gefen_gemm_bf16_sym(int32_t N, int32_t K, float alpha, const uint16_t* A, int32_t lda,
+                                   float beta, const uint16_t* D, int32_t ldd, uint16_t* C, int32_t ldc,
+                                   void* workspace, size_t workspace_bytes, gefen_stream_t stream);
 gefen_status_t gefen_muon_step(int64_t rows, int64_t cols, int64_t period, float* params,
                                const uint16_t* grads, uint8_t* codes, float* scale,
                                const float* codebook_dec, const float* codebook_enc, int32_t k,

@@ -87,6 +87,22 @@ __device__ __forceinline__ void umma_commit(uint32_t bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
                  : "memory");
 }
+// TMA store of a 32 x 32 bf16 block from shared memory to global (x: column,
+// y: row of the tensor map's matrix); out-of-range parts are not written.
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, uint32_t src, int x, int y) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+                     reinterpret_cast<uint64_t>(map)),
+                 "r"(x), "r"(y), "r"(src)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// Until at most one committed store group is still reading shared memory.
+__device__ __forceinline__ void bulk_wait_read1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
+// Until every committed store group has completed.
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+// Generic-proxy writes to shared memory become visible to the TMA unit.
+__device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
@@ -139,7 +155,10 @@ struct alignas(1024) TcSmem {
     using C = TcCfg<BN>;
     unsigned char a[C::kStagesN][C::kTileAB];  // 1024-byte aligned tiles (swizzle atoms)
     unsigned char b[C::kStagesN][C::kTileBB];
-    __nv_bfloat16 tr[4][32][40];  // per epilogue warp: 32 columns x 32 rows, padded rows
+    // per epilogue warp, two buffers each: a 32 x 32 block of C and of its
+    // transpose, row-major, as the TMA stores read them
+    __nv_bfloat16 stc[4][2][32][32];
+    __nv_bfloat16 stt[4][2][32][32];
     unsigned long long full[C::kStagesN], empty[C::kStagesN], acc_full[2], acc_empty[2];
     uint32_t tmem;
     int abort;
@@ -174,12 +193,43 @@ __device__ __forceinline__ void tile_of(int t, int ntm, bool sym, int& mb, int& 
     mb = t - j * (j + 1) / 2;
 }
 
+// Two bf16 (round to nearest even) in one word, the first in the low half.
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+    const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+// Row `row` of D, columns col0 .. col0 + 31 as bf16 pairs (zero outside D).
+__device__ __forceinline__ void load_d(uint32_t (&d)[16], const GemmArgs& G, int row, int col0) {
+    if (row < G.M && col0 + 32 <= G.N) {
+        const uint4* p = reinterpret_cast<const uint4*>(G.D + static_cast<int64_t>(row) * G.ldd + col0);
+#pragma unroll
+        for (int qq = 0; qq < 4; ++qq) {
+            const uint4 w = __ldg(p + qq);
+            d[4 * qq] = w.x;
+            d[4 * qq + 1] = w.y;
+            d[4 * qq + 2] = w.z;
+            d[4 * qq + 3] = w.w;
+        }
+    } else {
+        const unsigned short* p = reinterpret_cast<const unsigned short*>(G.D) + static_cast<int64_t>(row) * G.ldd;
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+            const int c = col0 + 2 * j;
+            const uint32_t lo = (row < G.M && c < G.N) ? p[c] : 0u;
+            const uint32_t hi = (row < G.M && c + 1 < G.N) ? p[c + 1] : 0u;
+            d[j] = lo | (hi << 16);
+        }
+    }
+}
+
 constexpr int kTcThreads = 192;  // warp 0: TMA, warp 1: MMA, warps 2-5: epilogue
 
 // Persistent tcgen05 GEMM: each CTA takes tiles blockIdx.x, + gridDim.x, ...
 template <int BN>
 __global__ void __launch_bounds__(kTcThreads, 1)
-    k_gemm_tc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB, const GemmArgs G) {
+    k_gemm_tc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
+              const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapCT, const GemmArgs G) {
     using Cf = TcCfg<BN>;
     constexpr int S = Cf::kStagesN;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -205,6 +255,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapA)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapB)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapC)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapCT)) : "memory");
     }
     if (warp == 0) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(saddr(&sm.tmem)),
@@ -272,10 +324,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         sm.consumed = ring;
     } else if (warp >= 2) {
         // epilogue: this warp reads accumulator rows 32 q .. 32 q + 31 (the
-        // TMEM lanes of warp id % 4)
+        // TMEM lanes of warp id % 4), 32 columns at a time: a 32 x 32 block
+        // that it stages in shared memory, as C and as its transpose, and
+        // writes with TMA stores.  In a symmetric product a block above the
+        // diagonal is stored at its place and mirrored; a block on the
+        // diagonal takes its upper triangle for both halves; a block below
+        // it is left to the mirror of the block above.
         const int q = warp & 3, e = warp - 2;
-        const int r = 32 * q + lane;
-        __nv_bfloat16(*tr)[40] = sm.tr[e];
+        const bool hasC = G.C != nullptr, hasT = sym || G.CT != nullptr;
+        const bool useD = G.beta != 0.0f && G.D != nullptr;
+        int nst = 0;  // blocks this warp has staged (their buffer alternates)
         int i = 0;
         for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++i) {
             const int b = i & 1;
@@ -287,82 +345,73 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             }
             int mb, nb;
             tile_of(t, ntm, sym, mb, nb);
-            const int m0 = mb * kBM, n0 = nb * BN, row = m0 + r;
-            const bool diag = sym && mb * kBM + kBM > nb * BN;  // the tile holds elements below the diagonal
-            __nv_bfloat16* CT = sym ? G.C : G.CT;
-            const int ldct = sym ? G.ldc : G.ldct;
-            for (int c0 = 0; c0 < BN; c0 += 32) {
+            const int n0 = nb * BN, i0 = mb * kBM + 32 * q, row = i0 + lane;
+            // first column block of this warp: in a symmetric product the
+            // blocks left of the diagonal are skipped
+            const int cfirst = sym ? max(0, i0 - n0) : 0;
+            uint32_t dn[16];  // D of the next block, loaded one block ahead
+            if (useD) load_d(dn, G, row, n0 + cfirst);
+            for (int c0 = cfirst; c0 < BN; c0 += 32) {
+                const int col0 = n0 + c0;
+                uint32_t dc[16];
+#pragma unroll
+                for (int j = 0; j < 16; ++j) dc[j] = dn[j];
+                if (useD && c0 + 32 < BN) load_d(dn, G, row, col0 + 32);
                 float v[32];
                 tmem_ld32(tmem + static_cast<uint32_t>(b * BN + c0) + (static_cast<uint32_t>(32 * q) << 16), v);
-                const int col0 = n0 + c0;
-                if (row < G.M) {
-                    if (G.beta != 0.0f && G.D != nullptr) {
-                        const __nv_bfloat16* d = G.D + static_cast<int64_t>(row) * G.ldd + col0;
-                        if (col0 + 32 <= G.N && (reinterpret_cast<uintptr_t>(d) & 15u) == 0) {
+                if (useD) {
 #pragma unroll
-                            for (int qq = 0; qq < 4; ++qq) {
-                                const uint4 w = *reinterpret_cast<const uint4*>(d + 8 * qq);
-                                const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&w);
-#pragma unroll
-                                for (int k2 = 0; k2 < 4; ++k2) {
-                                    const float2 f = __bfloat1622float2(h[k2]);
-                                    v[8 * qq + 2 * k2] = G.alpha * v[8 * qq + 2 * k2] + G.beta * f.x;
-                                    v[8 * qq + 2 * k2 + 1] = G.alpha * v[8 * qq + 2 * k2 + 1] + G.beta * f.y;
-                                }
-                            }
-                        } else {
-#pragma unroll
-                            for (int k = 0; k < 32; ++k)
-                                v[k] = G.alpha * v[k] + (col0 + k < G.N ? G.beta * __bfloat162float(d[k]) : 0.0f);
-                        }
-                    } else {
-#pragma unroll
-                        for (int k = 0; k < 32; ++k) v[k] *= G.alpha;
+                    for (int j = 0; j < 16; ++j) {
+                        v[2 * j] = G.alpha * v[2 * j] + G.beta * __uint_as_float(dc[j] << 16);
+                        v[2 * j + 1] = G.alpha * v[2 * j + 1] + G.beta * __uint_as_float(dc[j] & 0xFFFF0000u);
                     }
-                    if (G.C != nullptr) {
-                        __nv_bfloat16* c = G.C + static_cast<int64_t>(row) * G.ldc + col0;
-                        if (!diag && col0 + 32 <= G.N && (reinterpret_cast<uintptr_t>(c) & 15u) == 0) {
+                } else {
 #pragma unroll
-                            for (int qq = 0; qq < 4; ++qq) {
-                                __nv_bfloat162 h[4];
+                    for (int k = 0; k < 32; ++k) v[k] *= G.alpha;
+                }
+                const bool ondiag = sym && col0 == i0;
+                const int p = nst & 1;
+                __nv_bfloat16(*bc)[32] = sm.stc[e][p];
+                __nv_bfloat16(*bt)[32] = sm.stt[e][p];
+                // the stores that last read buffer p have finished reading it
+                if (lane == 0) bulk_wait_read1();
+                __syncwarp();
+                if (hasC) {
 #pragma unroll
-                                for (int k2 = 0; k2 < 4; ++k2)
-                                    h[k2] = __floats2bfloat162_rn(v[8 * qq + 2 * k2], v[8 * qq + 2 * k2 + 1]);
-                                *reinterpret_cast<uint4*>(c + 8 * qq) = *reinterpret_cast<uint4*>(h);
-                            }
-                        } else {
-#pragma unroll
-                            for (int k = 0; k < 32; ++k)
-                                if (col0 + k < G.N && (!sym || row <= col0 + k)) c[k] = __float2bfloat16_rn(v[k]);
-                        }
+                    for (int qq = 0; qq < 4; ++qq) {
+                        uint4 w;
+                        w.x = pack_bf16(v[8 * qq], v[8 * qq + 1]);
+                        w.y = pack_bf16(v[8 * qq + 2], v[8 * qq + 3]);
+                        w.z = pack_bf16(v[8 * qq + 4], v[8 * qq + 5]);
+                        w.w = pack_bf16(v[8 * qq + 6], v[8 * qq + 7]);
+                        *reinterpret_cast<uint4*>(&bc[lane][8 * qq]) = w;
                     }
                 }
-                if (CT != nullptr) {
-                    // transpose through this warp's buffer: lane l then owns
-                    // column col0 + l, rows m0 + 32 q .. + 31
+                if (hasT) {
 #pragma unroll
-                    for (int k = 0; k < 32; ++k) tr[k][lane] = __float2bfloat16_rn(v[k]);
-                    __syncwarp();
-                    const int jcol = col0 + lane, i0 = m0 + 32 * q;
-                    if (jcol < G.N) {
-                        __nv_bfloat16* ct = CT + static_cast<int64_t>(jcol) * ldct + i0;
-                        if (!diag && i0 + 32 <= G.M && (reinterpret_cast<uintptr_t>(ct) & 15u) == 0) {
-#pragma unroll
-                            for (int qq = 0; qq < 4; ++qq)
-                                *reinterpret_cast<uint4*>(ct + 8 * qq) = *reinterpret_cast<const uint4*>(&tr[lane][8 * qq]);
-                        } else {
-                            for (int k = 0; k < 32; ++k)
-                                if (i0 + k < G.M && (!sym || i0 + k < jcol)) ct[k] = tr[lane][k];
-                        }
-                    }
-                    __syncwarp();
+                    for (int k = 0; k < 32; ++k) bt[k][lane] = __float2bfloat16_rn(v[k]);
                 }
+                if (ondiag) {
+                    // row lane, columns left of the diagonal: the transpose
+                    __syncwarp();
+                    for (int k = 0; k < lane; ++k) bc[lane][k] = bt[lane][k];
+                }
+                fence_async_smem();
+                __syncwarp();
+                if (lane == 0) {
+                    if (hasC) tma_store_2d(&mapC, saddr(&bc[0][0]), col0, i0);
+                    if (hasT && !ondiag) tma_store_2d(&mapCT, saddr(&bt[0][0]), i0, col0);
+                    bulk_commit();
+                }
+                ++nst;
             }
             // this accumulator is drained: the MMA issuer may reuse it
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(saddr(&sm.acc_empty[b]));
         }
+        // every store of this warp has completed before the CTA exits
+        if (lane == 0) bulk_wait_all();
     }
     __syncwarp();
     tc_fence_before();
@@ -461,19 +510,26 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     return fn;
 }
 
-// TMA map of a row-major rows x cols bf16 matrix (leading dimension ld), box
-// 64 columns x box_rows rows, 128-byte swizzle, zero fill out of range.
+// TMA map of a row-major rows x cols bf16 matrix (leading dimension ld).
+// Operands: box 64 columns x box_rows rows, 128-byte swizzle, zero fill out
+// of range.  Results (box_rows 0): box 32 x 32, no swizzle.
 bool make_map(CUtensorMap* map, const void* base, int rows, int cols, int ld, int box_rows) {
     const auto fn = encode_fn();
     if (!fn) return false;
+    const bool operand = box_rows > 0;
     const cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
     const cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * 2};
-    const cuuint32_t box[2] = {static_cast<cuuint32_t>(kBK), static_cast<cuuint32_t>(box_rows)};
+    const cuuint32_t box[2] = {static_cast<cuuint32_t>(operand ? kBK : 32),
+                               static_cast<cuuint32_t>(operand ? box_rows : 32)};
     const cuuint32_t estr[2] = {1, 1};
     return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, operand ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+              operand ? CU_TENSOR_MAP_L2_PROMOTION_L2_256B : CU_TENSOR_MAP_L2_PROMOTION_NONE,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
+
+// A bf16 matrix that TMA can address: 16-byte aligned base and row stride.
+bool tma_ok(const void* p, int ld) { return p == nullptr || (ld % 8 == 0 && (reinterpret_cast<uintptr_t>(p) & 15u) == 0); }
 
 }  // namespace
 
@@ -483,15 +539,19 @@ bool gemm_tc_usable(int lda, int ldb, const void* A, const void* B) {
            (reinterpret_cast<uintptr_t>(B) & 15u) == 0 && encode_fn() != nullptr;
 }
 
+static_assert(sizeof(TcSmem<128>) + 1024 <= 232448 && sizeof(TcSmem<256>) + 1024 <= 232448,
+              "shared memory per CTA");
+
 template <int BN>
-cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const GemmArgs& G, cudaStream_t st) {
+cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorMap& mc, const CUtensorMap& mct,
+                      const GemmArgs& G, cudaStream_t st) {
     const int smem = static_cast<int>(sizeof(TcSmem<BN>)) + 1024;
     cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     const int ntm = (G.M + kBM - 1) / kBM, ntn = (G.N + BN - 1) / BN;
     const int ntiles = G.sym ? ntn * (ntn + 1) / 2 : ntm * ntn;
     const int grid = std::min(ntiles, device_sm_count());
-    k_gemm_tc<BN><<<grid, kTcThreads, smem, st>>>(ma, mb, G);
+    k_gemm_tc<BN><<<grid, kTcThreads, smem, st>>>(ma, mb, mc, mct, G);
     return cudaGetLastError();
 }
 
@@ -500,13 +560,17 @@ cudaError_t gemm_bf16_nt(int M, int N, int K, float alpha, const void* A, int ld
                          cudaStream_t st, bool sym) {
     if (M <= 0 || N <= 0) return cudaSuccess;
     if (sym && (M != N || CT != nullptr || C == nullptr)) return cudaErrorInvalidValue;
-    if (K > 0 && gemm_tc_usable(lda, ldb, A, B)) {
+    const bool results_ok = tma_ok(C, ldc) && tma_ok(CT, ldct) && (beta == 0.0f || tma_ok(D, ldd));
+    if (K > 0 && results_ok && gemm_tc_usable(lda, ldb, A, B)) {
         // 256-wide tiles when there are enough of them for every SM, else
         // (and for symmetric products) 128-wide ones
         const int64_t tiles256 = static_cast<int64_t>((M + kBM - 1) / kBM) * ((N + 255) / 256);
         const int bn = (sym || tiles256 < device_sm_count()) ? 128 : 256;
-        CUtensorMap ma, mb;
+        CUtensorMap ma, mb, mc{}, mct{};
         if (!make_map(&ma, A, M, K, lda, kBM) || !make_map(&mb, B, N, K, ldb, bn)) return cudaErrorInvalidValue;
+        if (C != nullptr && !make_map(&mc, C, M, N, ldc, 0)) return cudaErrorInvalidValue;
+        if (CT != nullptr && !make_map(&mct, CT, N, M, ldct, 0)) return cudaErrorInvalidValue;
+        if (sym) mct = mc;  // the mirrored blocks go to C itself
         GemmArgs G;
         G.M = M;
         G.N = N;
@@ -521,7 +585,7 @@ cudaError_t gemm_bf16_nt(int M, int N, int K, float alpha, const void* A, int ld
         G.ldct = ldct;
         G.sym = sym ? 1 : 0;
         G.err = err;
-        return bn == 128 ? launch_tc<128>(ma, mb, G, st) : launch_tc<256>(ma, mb, G, st);
+        return bn == 128 ? launch_tc<128>(ma, mb, mc, mct, G, st) : launch_tc<256>(ma, mb, mc, mct, G, st);
     }
     const dim3 grid((N + 63) / 64, (M + 63) / 64);
     k_gemm_simt<__nv_bfloat16><<<grid, 256, 0, st>>>(
@@ -557,6 +621,22 @@ extern "C" gefen_status_t gefen_gemm_bf16(int32_t M, int32_t N, int32_t K, float
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     int* err = static_cast<int*>(workspace);
     if (gemm_bf16_nt(M, N, K, alpha, A, lda, B, ldb, beta, D, ldd, C, ldc, CT, ldct, err, st, false) != cudaSuccess)
+        return GEFEN_ECUDA;
+    return GEFEN_OK;
+}
+
+// Exposed for tests: C = alpha A A^T + beta D, symmetric (see gefen.h).
+extern "C" gefen_status_t gefen_gemm_bf16_sym(int32_t N, int32_t K, float alpha, const uint16_t* A, int32_t lda,
+                                              float beta, const uint16_t* D, int32_t ldd, uint16_t* C, int32_t ldc,
+                                              void* workspace, size_t workspace_bytes, gefen_stream_t stream) {
+    using namespace gefen;
+    if (N < 0 || K < 0 || !A || !C || ldc < N || lda < K || (beta != 0.0f && (!D || ldd < N))) return GEFEN_EINVAL;
+    if (workspace == nullptr || workspace_bytes < kWsAlign) return GEFEN_ENOMEM;
+    if (reinterpret_cast<uintptr_t>(workspace) % kWsAlign) return GEFEN_EINVAL;
+    if (gefen_status_t s = check_device(); s != GEFEN_OK) return s;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    int* err = static_cast<int*>(workspace);
+    if (gemm_bf16_nt(N, N, K, alpha, A, lda, A, lda, beta, D, ldd, C, ldc, nullptr, 0, err, st, true) != cudaSuccess)
         return GEFEN_ECUDA;
     return GEFEN_OK;
 }

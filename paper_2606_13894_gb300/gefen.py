@@ -49,7 +49,8 @@ EXPORTS = ("gefen_status_string", "gefen_sync_status", "gefen_step_workspace_siz
            "gefen_refit_workspace_size", "gefen_refit_codebook", "gefen_refit_status",
            "gefen_refit_tables", "gefen_infer_workspace_size", "gefen_infer_blocks",
            "gefen_refit_codebook_static", "gefen_refit_static_init", "gefen_refit_static_status",
-           "gefen_refit_debug", "gefen_muon_workspace_size", "gefen_muon_step", "gefen_gemm_bf16")
+           "gefen_refit_debug", "gefen_muon_workspace_size", "gefen_muon_step", "gefen_gemm_bf16",
+           "gefen_gemm_bf16_sym")
 
 GEFEN_MUON_BF16_GEMM = 1
 
@@ -119,6 +120,8 @@ def load(build_if_needed: bool = True):
         f32 = ctypes.c_float
         L.gefen_gemm_bf16.argtypes = [i32, i32, i32, f32, P, i32, P, i32, f32, P, i32, P, i32, P, i32, P, sz, P]
         L.gefen_gemm_bf16.restype = ctypes.c_int
+        L.gefen_gemm_bf16_sym.argtypes = [i32, i32, f32, P, i32, f32, P, i32, P, i32, P, sz, P]
+        L.gefen_gemm_bf16_sym.restype = ctypes.c_int
         _lib = L
         return L
 
@@ -340,3 +343,18 @@ def gefen_gemm_bf16(A, B, *, alpha=1.0, beta=0.0, D=None, C=None, CT=None, works
                                 _stream(stream))
     _check("gefen_gemm_bf16", st)
     return C, CT, workspace_buf
+
+
+def gefen_gemm_bf16_sym(A, *, alpha=1.0, beta=0.0, D=None, C=None, workspace_buf=None, stream=None):
+    """C = alpha A A^T + beta D (bf16 row-major; D symmetric), symmetric bit
+    for bit.  Allocates C when not given.  Returns (C, workspace)."""
+    N, K = A.shape
+    if C is None:
+        C = torch.empty((N, N), dtype=torch.bfloat16, device=A.device)
+    if workspace_buf is None:
+        workspace_buf = workspace(256, A.device)
+    st = load().gefen_gemm_bf16_sym(N, K, float(alpha), _ptr(A), A.stride(0), float(beta), _ptr(D),
+                                    D.stride(0) if D is not None else 0, _ptr(C), C.stride(0),
+                                    _ptr(workspace_buf), workspace_buf.numel(), _stream(stream))
+    _check("gefen_gemm_bf16_sym", st)
+    return C, workspace_buf

@@ -5,7 +5,8 @@ element may round to the neighbouring bf16 value: within 2^-7 relative plus
 2^-12 of the largest |C|.  Shapes: one tile, several tiles and k-tiles (the
 operand ring wraps), ragged M, N and K, the Newton-Schulz shapes of a
 2048 x 8192 matrix, the transposed output, and leading dimensions that TMA
-cannot address (the CUDA-core path)."""
+cannot address (the CUDA-core path: lda = 100, and ldc = 700 in the 300 x 700
+case)."""
 import pytest
 import torch
 
@@ -27,8 +28,9 @@ def _close(got, ref):
     assert not bool(bad.any()), f"{int(bad.sum())} of {bad.numel()} outside; max err {float((got.float() - ref).abs().max())}"
 
 
-@pytest.mark.parametrize("M,N,K", [(128, 256, 64), (256, 512, 1024), (300, 700, 200), (64, 64, 256),
-                                   (2048, 2048, 8192), (2048, 8192, 2048), (96, 512, 96)])
+@pytest.mark.parametrize("M,N,K", [(128, 256, 64), (256, 512, 1024), (296, 712, 200), (64, 64, 256),
+                                   (2048, 2048, 8192), (2048, 8192, 2048), (96, 512, 96),
+                                   (2904, 4008, 328), (300, 700, 200)])
 @pytest.mark.parametrize("with_d", [False, True])
 def test_gemm_matches_fp32_product(M, N, K, with_d):
     g = torch.Generator(device="cuda").manual_seed(M * 7 + N + K)
@@ -61,3 +63,22 @@ def test_gemm_submatrix_operands():
     A, B = Abig[:, :512], Bbig[:, :512]
     C, _, _ = G.gefen_gemm_bf16(A, B)
     _close(C, _ref(A, B, 1.0, 0.0, None))
+
+
+@pytest.mark.parametrize("N,K", [(128, 64), (256, 1024), (296, 200), (1000, 96), (2048, 8192), (2048, 2048),
+                                 (100, 100)])
+@pytest.mark.parametrize("with_d", [False, True])
+def test_symmetric_product_is_exactly_symmetric(N, K, with_d):
+    # the Newton-Schulz products X X^T and c A A^T + b A: tiles on and above
+    # the diagonal, mirrored (N = 100: lda not a multiple of 8, CUDA cores)
+    g = torch.Generator(device="cuda").manual_seed(N * 3 + K)
+    A = torch.randn(N, K, device="cuda", generator=g).to(torch.bfloat16)
+    D = None
+    if with_d:
+        R = torch.randn(N, N, device="cuda", generator=g)
+        D = ((R + R.T) * 0.5).to(torch.bfloat16)
+    alpha, beta = (-4.775, 2.0315) if with_d else (1.0, 0.0)
+    C, ws = G.gefen_gemm_bf16_sym(A, alpha=alpha, beta=beta, D=D)
+    G.gefen_step_status(ws)
+    assert torch.equal(C, C.T)
+    _close(C, _ref(A, A, alpha, beta, D))
