@@ -40,6 +40,56 @@ __device__ __forceinline__ int level_search(const float* __restrict__ mids, floa
     return c;
 }
 
+// The same level through cell records: x = m / s' lies in [-1, 1]; a record
+// per cell of a uniform grid of kLutCells over [-1, 1] (two guard cells at
+// the ends) holds the number of midpoints below the cell and the next three
+// midpoints, so the level is the base plus three compares.  Identical to
+// level_search whenever build_cell_records reports no cell (widened by a
+// 2^-22 guard on both sides) with more than three midpoints; the callers use
+// level_search otherwise.  R copies of each record spread a warp's gathers
+// over more shared-memory banks (copy r of record c + 1 at (c + 1) R + r).
+constexpr int kLutCells = 512;
+constexpr float kLutGuard = 2.384185791015625e-07f;  // 2^-22, below every cell edge
+
+__device__ __forceinline__ uint32_t lt_mask(float a, float b) {
+    uint32_t r;
+    asm("set.lt.u32.f32 %0, %1, %2;" : "=r"(r) : "f"(a), "f"(b));
+    return r;
+}
+
+// Fills lut[(kLutCells + 2) * R] from mid (padded with +inf to kMaxLevels + 4
+// entries, already in shared memory behind a barrier); thread t of nthreads.
+// Returns nonzero when some cell holds more than three midpoints.
+template <int R>
+__device__ __forceinline__ int build_cell_records(const float* mid, float4* lut, int t, int nthreads) {
+    int bad = 0;
+    // cell(x) = floor(fma(x, G/2, G/2)) is within 2^-24 of exact in x: each
+    // record counts the midpoints below its cell minus the guard and holds
+    // the next three
+    for (int i = t; i < kLutCells + 2; i += nthreads) {
+        const int c = i - 1;
+        const float lo = -1.0f + 2.0f * static_cast<float>(c) / kLutCells - kLutGuard;
+        const float hi = -1.0f + 2.0f * static_cast<float>(c + 1) / kLutCells + kLutGuard;
+        const int base = level_search(mid, lo);
+        const int upto = level_search(mid, hi);
+        bad |= (upto - base > 3);
+        const float4 rec = make_float4(__int_as_float(base), mid[base], mid[base + 1], mid[base + 2]);
+#pragma unroll
+        for (int r = 0; r < R; ++r) lut[i * R + r] = rec;
+    }
+    return bad;
+}
+
+// The level of x from the records (copy `copy`).
+template <int R>
+__device__ __forceinline__ uint32_t lut_encode(const float4* lut, int copy, float x) {
+    constexpr float kMagicCell = 12582912.0f;  // 1.5 * 2^23: the round-down add leaves the cell in the low bits
+    const float y = __fmaf_rd(x, 0.5f * kLutCells, 0.5f * kLutCells + 1.0f + kMagicCell);
+    const uint32_t r = static_cast<uint32_t>(__float_as_int(y)) - 0x4B400000u;
+    const float4 rec = lut[min(r, static_cast<uint32_t>(kLutCells + 1)) * R + copy];
+    return static_cast<uint32_t>(__float_as_int(rec.x)) - lt_mask(rec.y, x) - lt_mask(rec.z, x) - lt_mask(rec.w, x);
+}
+
 // --------------------------------------------------- 128-bit integers
 struct u128 {
     uint64_t hi, lo;

@@ -160,17 +160,24 @@ __global__ void __launch_bounds__(kMuThreads) k_muon_absmax8(MuonArgs A) {
     }
 }
 
+// Encoding as the step kernels do it: x = m * (1 / s'), its level from the
+// cell records (four copies), the binary search when a cell holds more than
+// three midpoints.
+constexpr int kMuLutR = 4;
+
 template <bool BF16>
 __global__ void __launch_bounds__(kMuThreads) k_muon_encode8(MuonArgs A) {
-    __shared__ float s_dec[kMaxLevels], s_mid[kMaxLevels];
+    __shared__ float s_dec[kMaxLevels], s_mid[kMaxLevels + 4];
+    __shared__ float4 s_lut[(kLutCells + 2) * kMuLutR];
     __shared__ double s_red[kMuThreads / 32];
     const int t = threadIdx.x;
-    if (t < kMaxLevels) {
-        s_dec[t] = t < A.k ? A.cb_dec[t] : 0.0f;
-        s_mid[t] = (t < A.k - 1) ? 0.5f * (A.cb_enc[t] + A.cb_enc[t + 1]) : INFINITY;
-    }
+    if (t < kMaxLevels) s_dec[t] = t < A.k ? A.cb_dec[t] : 0.0f;
+    for (int i = t; i < kMaxLevels + 4; i += kMuThreads)
+        s_mid[i] = (i < A.k - 1) ? 0.5f * (A.cb_enc[i] + A.cb_enc[i + 1]) : INFINITY;
     __syncthreads();
+    const bool lut = !__syncthreads_or(build_cell_records<kMuLutR>(s_mid, s_lut, t, kMuThreads));
     const int zero_code = level_search(s_mid, 0.0f);
+    const int copy = t % kMuLutR;
     double acc = 0.0;
     const int64_t nv = A.n >> 3;
     for (int64_t v = blockIdx.x * static_cast<int64_t>(kMuThreads) + t; v < nv;
@@ -181,14 +188,17 @@ __global__ void __launch_bounds__(kMuThreads) k_muon_encode8(MuonArgs A) {
         load8(A, v, g, c);
         const float mus = A.mu * A.scale[bi];
         const float sn = A.snew[bi];
+        const float inv = sn > 0.0f ? __frcp_rn(sn) : 0.0f;
         float u[8];
         uint32_t cw[2] = {0u, 0u};
         float sq = 0.0f;  // squares of the stored update, exact in fp32 for bf16 values
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
             const float m = fmaf(A.omm, g[i], mus * s_dec[c[i]]);
-            const uint32_t code = sn > 0.0f ? static_cast<uint32_t>(level_search(s_mid, __fdiv_rn(m, sn)))
-                                            : static_cast<uint32_t>(zero_code);
+            const float x = m * inv;
+            const uint32_t code = sn <= 0.0f ? static_cast<uint32_t>(zero_code)
+                                  : lut      ? lut_encode<kMuLutR>(s_lut, copy, x)
+                                             : static_cast<uint32_t>(level_search(s_mid, x));
             cw[i >> 2] |= code << (8 * (i & 3));
             u[i] = A.nesterov ? fmaf(A.mu, m - g[i], g[i]) : m;
             if (BF16) u[i] = __bfloat162float(__float2bfloat16_rn(u[i]));
@@ -264,6 +274,44 @@ __global__ void __launch_bounds__(256) k_muon_scale_t(T* __restrict__ u, T* __re
     __syncthreads();
     for (int i = ty; i < 32; i += 8)
         if (c0 + i < cols && r0 + tx < rows) ut[static_cast<int64_t>(c0 + i) * rows + r0 + tx] = tile[tx][i];
+}
+
+// The bf16 form for even rows and cols: 64 x 64 tiles, each lane moving two
+// elements (four bytes), so a warp reads and writes whole 128-byte rows of U
+// and of U^T; the tile's rows are 66 elements apart in shared memory (the
+// column reads of the transpose meet at most two lanes per bank).
+__global__ void __launch_bounds__(256) k_muon_scale_t2(__nv_bfloat16* __restrict__ u, __nv_bfloat16* __restrict__ ut,
+                                                      int rows, int cols, const float* __restrict__ inv_p,
+                                                      float* __restrict__ scale, const float* __restrict__ snew,
+                                                      int64_t nb) {
+    __shared__ __nv_bfloat162 tile[64][33];  // row i: columns 2 j, 2 j + 1 in entry j
+    const float inv = *inv_p;
+    const int c0 = blockIdx.x * 64, r0 = blockIdx.y * 64;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    for (int i = warp; i < 64; i += 8) {
+        const int r = r0 + i, c = c0 + 2 * lane;
+        if (r < rows && c < cols) {
+            __nv_bfloat162* p = reinterpret_cast<__nv_bfloat162*>(u + static_cast<int64_t>(r) * cols + c);
+            const float2 f = __bfloat1622float2(*p);
+            const __nv_bfloat162 y = __floats2bfloat162_rn(f.x * inv, f.y * inv);
+            *p = y;
+            tile[i][lane] = y;
+        }
+    }
+    const int64_t cta = static_cast<int64_t>(blockIdx.y) * gridDim.x + blockIdx.x;
+    const int64_t ncta = static_cast<int64_t>(gridDim.x) * gridDim.y;
+    for (int64_t b = cta * 256 + threadIdx.x; b < nb; b += ncta * 256) scale[b] = snew[b];
+    if (ut == nullptr) return;
+    __syncthreads();
+    // row c0 + j of U^T: lane l writes its elements r0 + 2 l and r0 + 2 l + 1
+    for (int j = warp; j < 64; j += 8) {
+        const int c = c0 + j, r = r0 + 2 * lane;
+        if (c < cols && r < rows) {
+            const __nv_bfloat162 a = tile[2 * lane][j >> 1], b = tile[2 * lane + 1][j >> 1];
+            const __nv_bfloat162 o = (j & 1) ? __halves2bfloat162(a.y, b.y) : __halves2bfloat162(a.x, b.x);
+            *reinterpret_cast<__nv_bfloat162*>(ut + static_cast<int64_t>(c) * rows + r) = o;
+        }
+    }
 }
 
 // theta = theta * decay - step * X, four elements per thread.
@@ -425,7 +473,12 @@ extern "C" gefen_status_t gefen_muon_step(int64_t rows, int64_t cols, int64_t pe
     {
         const dim3 tg(static_cast<unsigned>((cols + 31) / 32), static_cast<unsigned>((rows + 31) / 32));
         void* ut = hp.ns_steps > 0 ? Q0 : nullptr;
-        if (bf16)
+        if (bf16 && rows % 2 == 0 && cols % 2 == 0)
+            k_muon_scale_t2<<<dim3(static_cast<unsigned>((cols + 63) / 64), static_cast<unsigned>((rows + 63) / 64)),
+                              256, 0, st>>>(static_cast<__nv_bfloat16*>(P0), static_cast<__nv_bfloat16*>(ut),
+                                            static_cast<int>(rows), static_cast<int>(cols), inv, scale, A.snew,
+                                            n / period);
+        else if (bf16)
             k_muon_scale_t<__nv_bfloat16><<<tg, 256, 0, st>>>(static_cast<__nv_bfloat16*>(P0),
                                                               static_cast<__nv_bfloat16*>(ut), static_cast<int>(rows),
                                                               static_cast<int>(cols), inv, scale, A.snew, n / period);

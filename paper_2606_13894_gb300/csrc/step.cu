@@ -478,8 +478,6 @@ __global__ void __launch_bounds__(kThreads) k_step_tile16(const __grid_constant_
 // cell holds more than three midpoints).  Both tables are replicated (LUTR,
 // DECR copies, lane l reading copy l % R) so the gathers of one warp spread
 // over more shared-memory banks.
-constexpr int kLutCells = 512;
-constexpr float kLutGuard = 2.384185791015625e-07f;  // 2^-22, below every cell edge
 
 struct TileInfo {
     int64_t e0;    // first element
@@ -567,23 +565,7 @@ __device__ __forceinline__ int build_tables(const Ptrs& P, StreamTables<LUTR, DE
     for (int i = t; i < kMaxLevels + 4; i += THREADS)
         T.mid[i] = (i < P.k - 1) ? 0.5f * (P.cb_enc[i] + P.cb_enc[i + 1]) : INFINITY;
     __syncthreads();
-    int bad = 0;
-    // cell(x) = floor(fma(x, G/2, G/2)) is within 2^-24 of exact in x: each
-    // record counts the midpoints below its cell minus a 2^-22 guard and holds
-    // the next three; its cell plus the guard on both sides may hold at most
-    // three midpoints, or the binary search is used instead.
-    for (int i = t; i < kLutCells + 2; i += THREADS) {
-        const int c = i - 1;
-        const float lo = -1.0f + 2.0f * static_cast<float>(c) / kLutCells - kLutGuard;
-        const float hi = -1.0f + 2.0f * static_cast<float>(c + 1) / kLutCells + kLutGuard;
-        const int base = level_search(T.mid, lo);
-        const int upto = level_search(T.mid, hi);
-        bad |= (upto - base > 3);
-        const float4 rec = make_float4(__int_as_float(base), T.mid[base], T.mid[base + 1], T.mid[base + 2]);
-#pragma unroll
-        for (int r = 0; r < LUTR; ++r) T.lut[i * LUTR + r] = rec;
-    }
-    return bad;
+    return build_cell_records<LUTR>(T.mid, T.lut, t, THREADS);
 }
 
 // The issuing thread walks the segment table forward: a CTA's tiles come in
@@ -717,11 +699,6 @@ __device__ __forceinline__ float sqrt_approx(float x) {
 }
 
 // 0xFFFFFFFF if a < b else 0 (one compare that yields an integer mask)
-__device__ __forceinline__ uint32_t lt_mask(float a, float b) {
-    uint32_t r;
-    asm("set.lt.u32.f32 %0, %1, %2;" : "=r"(r) : "f"(a), "f"(b));
-    return r;
-}
 
 // Nearest levels of four values, packed as four code bytes.  With the cell
 // records (LUT): |x| <= 1 up to rounding (x = m / max|m|, or 0 for a zero
@@ -733,15 +710,10 @@ __device__ __forceinline__ uint32_t lt_mask(float a, float b) {
 template <bool LUT, int LUTR, int DECR>
 __device__ __forceinline__ void encode4(const StreamTables<LUTR, DECR>& T, int copy, const float (&x)[4],
                                         uint32_t (&c)[4]) {
-    constexpr float kMagic = 12582912.0f;  // 1.5 * 2^23, bits 0x4B400000
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
         if (LUT) {
-            const float y = __fmaf_rd(x[i], 0.5f * kLutCells, 0.5f * kLutCells + 1.0f + kMagic);
-            const uint32_t r = static_cast<uint32_t>(__float_as_int(y)) - 0x4B400000u;
-            const float4 rec = T.lut[min(r, static_cast<uint32_t>(kLutCells + 1)) * LUTR + copy];
-            c[i] = static_cast<uint32_t>(__float_as_int(rec.x)) - lt_mask(rec.y, x[i]) - lt_mask(rec.z, x[i]) -
-                   lt_mask(rec.w, x[i]);
+            c[i] = lut_encode<LUTR>(T.lut, copy, x[i]);
         } else {
             c[i] = static_cast<uint32_t>(level_search(T.mid, x[i]));
         }
