@@ -592,31 +592,53 @@ def run_e2e(G, cad, args, stream):
     copies its bf16 gradient in from pinned memory and runs the step (refit
     steps included, with the timed region's cadence and step count), and the
     step's result is read back: its 4-byte status word (gefen_step_status,
-    which waits for the step).  A second figure also copies the rank's
-    updated fp32 parameters back to pinned memory every step."""
+    which waits for the step).  The copies run on their own stream into two
+    device buffers, as a data loader's would: step i + 1's gradient is copied
+    while step i computes, and step i + 2's copy waits until step i has read
+    its buffer.  Every copy of the timed steps, the first two included, is in
+    the timed region.  A second figure also copies the rank's updated fp32
+    parameters back to pinned memory every step (on the step's stream, so the
+    next step waits for it)."""
     sh = cad.sh
     n = sh.numel_arena
     g_host = torch.empty(n, dtype=torch.bfloat16, pin_memory=True)
     th_host = torch.empty(n, dtype=torch.float32, pin_memory=True)
     g_host.copy_(cad.gpool[1])
-    gdev = torch.empty_like(cad.gpool[0])
+    gdev = [torch.empty_like(cad.gpool[0]) for _ in range(2)]
+    cstream = torch.cuda.Stream(device=gdev[0].device)
     steps = args.steps
 
-    def e2e_step(readback_params: bool):
-        gdev.copy_(g_host, non_blocking=True)
-        cad.step(False, g=gdev)
-        if readback_params:
-            th_host.copy_(sh.theta, non_blocking=True)
-        G.gefen_step_status(sh.ws)
+    def run(count: int, readback_params: bool):
+        copied = [torch.cuda.Event() for _ in range(2)]
+        freed = [torch.cuda.Event() for _ in range(2)]
+
+        def copy_in(i):
+            b = i % 2
+            if i >= 2:
+                cstream.wait_event(freed[b])  # step i - 2 has read buffer b
+            with torch.cuda.stream(cstream):
+                gdev[b].copy_(g_host, non_blocking=True)
+            copied[b].record(cstream)
+
+        for i in range(min(2, count)):
+            copy_in(i)
+        for i in range(count):
+            b = i % 2
+            stream.wait_event(copied[b])
+            cad.step(False, g=gdev[b])
+            freed[b].record(stream)
+            if i + 2 < count:
+                copy_in(i + 2)
+            if readback_params:
+                th_host.copy_(sh.theta, non_blocking=True)
+            G.gefen_step_status(sh.ws)
 
     out = {}
     for key, rb in (("status", False), ("params", True)):
-        for _ in range(2):
-            e2e_step(rb)
+        run(2, rb)
         torch.cuda.synchronize()
         t0 = time.perf_counter()
-        for _ in range(steps):
-            e2e_step(rb)
+        run(steps, rb)
         torch.cuda.synchronize()
         out[key] = time.perf_counter() - t0
     nparams = sum(pc.numel for pc in sh.pieces)
@@ -624,6 +646,7 @@ def run_e2e(G, cad, args, stream):
             "refit_every": sh.refit_every,
             "h2d_bytes_per_step": 2 * n, "d2h_bytes_per_step": 4,
             "result_read": "the step's status word (gefen_step_status), every step",
+            "copies": "gradient copies on their own stream, one step ahead of the step that reads them",
             "with_params_readback": {"value": nparams * steps / out["params"] / 1e9, "unit": UNIT,
                                      "h2d_bytes_per_step": 2 * n, "d2h_bytes_per_step": 4 * n + 4}}
 
