@@ -402,14 +402,17 @@ def run_gpu(args, world, rank, local):
         "metric": METRIC, "value": whole_job_value(nparams, args.steps, elapsed_ms), "unit": UNIT,
         "n_gpus": world, "steps": args.steps, "warmup": warm, "ms_per_step": elapsed_ms / args.steps,
         "higher_is_better": True, "scaling": "strong", "vs_baseline": None, "dtype": "f32",
-        "data": "synthetic (seeded; shapes and gradient-scale structure of the Llama-3-1.5B run)",
+        "data": f"synthetic (seeded; shapes and gradient-scale structure of the {args.workload} set)",
         "config": {"workload": f"{args.workload} shaped set: {len(specs)} tensors, {nparams} fp32 params, "
                                f"{nblocks} inferred blocks; 256-level codebook; refit every {REFIT_EVERY} "
                                f"steps with {BINS} cells (16 per level: Algorithm 3's 16k cells read as 16 k); "
                                f"the same job with 65536-cell refits is under refit_65536",
                    "params": nparams, "tensors": len(specs), "blocks": nblocks, "refit_every": REFIT_EVERY,
                    "bins": BINS, "levels": K, "hparams": HP,
-                   "l2": "inputs larger than L2: 17.7 GB of step traffic per step, no flush needed",
+                   "l2": (f"inputs larger than L2: {alg_bytes / 1e9:.2f} GB of step traffic per step against a "
+                          f"129 MB L2, no flush needed" if alg_bytes > 4 * 129e6 else
+                          f"{alg_bytes / 1e9:.3f} GB of step traffic per step against a 129 MB L2: timings "
+                          f"of this workload include L2 reuse between steps"),
                    "parallelism": ("single GPU" if world == 1 else
                                    f"block-sharded over {world} ranks ({n_rank} params on rank {rank}); "
                                    f"one histogram all-reduce per refit")},
