@@ -133,6 +133,7 @@ struct GemmArgs {
     __nv_bfloat16* CT;
     int ldct;
     int sym;  // C is symmetric (M == N): only tiles on or above the diagonal are computed, each written twice
+    int nfull;  // tiles taken whole; the rest (a last, partial wave) as two halves of BN / 2 columns each
     int* err;
 };
 
@@ -148,6 +149,10 @@ struct TcCfg {
     static constexpr uint32_t kIdescN = (1u << 4) | (1u << 7) | (1u << 10) |
                                         (static_cast<uint32_t>(BN >> 3) << 17) |
                                         (static_cast<uint32_t>(kBM >> 4) << 24);
+    // the same with N = BN / 2 (half tiles)
+    static constexpr uint32_t kIdescHalf = (1u << 4) | (1u << 7) | (1u << 10) |
+                                           (static_cast<uint32_t>(BN >> 4) << 17) |
+                                           (static_cast<uint32_t>(kBM >> 4) << 24);
 };
 
 template <int BN>
@@ -223,13 +228,32 @@ __device__ __forceinline__ void load_d(uint32_t (&d)[16], const GemmArgs& G, int
     }
 }
 
+// Work item `it` of the schedule: a whole tile (it < nfull, and every tile of
+// a symmetric product) or one half of a tile of the last wave, BN / 2 columns
+// wide.  Gives its row block, first column and width.
+template <int BN>
+__device__ __forceinline__ void item_of(int it, int ntm, bool sym, int nfull, int& mb, int& n0, int& ncols) {
+    int nb;
+    if (sym || it < nfull) {
+        tile_of(it, ntm, sym, mb, nb);
+        n0 = nb * BN;
+        ncols = BN;
+    } else {
+        const int h = it - nfull;
+        tile_of(nfull + (h >> 1), ntm, false, mb, nb);
+        n0 = nb * BN + (h & 1) * (BN / 2);
+        ncols = BN / 2;
+    }
+}
+
 constexpr int kTcThreads = 192;  // warp 0: TMA, warp 1: MMA, warps 2-5: epilogue
 
 // Persistent tcgen05 GEMM: each CTA takes tiles blockIdx.x, + gridDim.x, ...
 template <int BN>
 __global__ void __launch_bounds__(kTcThreads, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
-              const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapCT, const GemmArgs G) {
+              const __grid_constant__ CUtensorMap mapBh, const __grid_constant__ CUtensorMap mapC,
+              const __grid_constant__ CUtensorMap mapCT, const GemmArgs G) {
     using Cf = TcCfg<BN>;
     constexpr int S = Cf::kStagesN;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -240,6 +264,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const int ntm = (G.M + kBM - 1) / kBM, ntn = (G.N + BN - 1) / BN;
     const bool sym = G.sym != 0;
     const int ntiles = sym ? ntn * (ntn + 1) / 2 : ntm * ntn;
+    const int nfull = sym ? ntiles : G.nfull;
+    const int nitems = nfull + 2 * (ntiles - nfull);
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
@@ -255,6 +281,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapA)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapB)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapBh)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapC)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&mapCT)) : "memory");
     }
@@ -274,9 +301,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (threadIdx.x == 0) {
         // producer: the A and B k-tiles of every tile of this CTA, in order
         int ring = 0;
-        for (int t = blockIdx.x; t < ntiles && !*abort; t += gridDim.x) {
-            int mb, nb;
-            tile_of(t, ntm, sym, mb, nb);
+        for (int t = blockIdx.x; t < nitems && !*abort; t += gridDim.x) {
+            int mb, n0, ncols;
+            item_of<BN>(t, ntm, sym, nfull, mb, n0, ncols);
+            const bool whole = ncols == BN;
             for (int kt = 0; kt < KT; ++kt, ++ring) {
                 const int s = ring % S;
                 if (ring >= S && !mbar_wait(saddr(&sm.empty[s]), static_cast<uint32_t>((ring / S - 1) & 1))) {
@@ -284,9 +312,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     break;
                 }
                 const uint32_t bar = saddr(&sm.full[s]);
-                mbar_expect_tx(bar, Cf::kTileAB + Cf::kTileBB);
+                mbar_expect_tx(bar, Cf::kTileAB + (whole ? Cf::kTileBB : Cf::kTileBB / 2));
                 tma_load_2d(saddr(sm.a[s]), &mapA, kt * kBK, mb * kBM, bar);
-                tma_load_2d(saddr(sm.b[s]), &mapB, kt * kBK, nb * BN, bar);
+                tma_load_2d(saddr(sm.b[s]), whole ? &mapB : &mapBh, kt * kBK, n0, bar);
                 issued = ring + 1;
             }
         }
@@ -294,7 +322,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         // MMA issuer: accumulator b = i & 1 for the CTA's i-th tile, reused
         // once the epilogue has drained it
         int ring = 0, i = 0;
-        for (int t = blockIdx.x; t < ntiles && !*abort; t += gridDim.x, ++i) {
+        for (int t = blockIdx.x; t < nitems && !*abort; t += gridDim.x, ++i) {
+            const uint32_t idesc = (sym || t < nfull) ? Cf::kIdescN : Cf::kIdescHalf;
             const int b = i & 1;
             if (i >= 2 && !mbar_wait(saddr(&sm.acc_empty[b]), static_cast<uint32_t>(((i >> 1) - 1) & 1))) {
                 atomicExch(&sm.abort, 1);
@@ -314,7 +343,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 const uint32_t a0 = saddr(sm.a[s]), b0 = saddr(sm.b[s]);
 #pragma unroll
                 for (int kk = 0; kk < kBK / 16; ++kk)
-                    umma_bf16_n(acc, desc_sw128(a0 + kk * 32), desc_sw128(b0 + kk * 32), Cf::kIdescN,
+                    umma_bf16_n(acc, desc_sw128(a0 + kk * 32), desc_sw128(b0 + kk * 32), idesc,
                                 (kt | kk) != 0 ? 1u : 0u);
                 umma_commit(saddr(&sm.empty[s]));
             }
@@ -335,7 +364,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const bool useD = G.beta != 0.0f && G.D != nullptr;
         int nst = 0;  // blocks this warp has staged (their buffer alternates)
         int i = 0;
-        for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++i) {
+        for (int t = blockIdx.x; t < nitems; t += gridDim.x, ++i) {
             const int b = i & 1;
             const bool ok = mbar_wait(saddr(&sm.acc_full[b]), static_cast<uint32_t>((i >> 1) & 1));
             tc_fence_after();
@@ -343,20 +372,20 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 atomicExch(&sm.abort, 1);
                 break;
             }
-            int mb, nb;
-            tile_of(t, ntm, sym, mb, nb);
-            const int n0 = nb * BN, i0 = mb * kBM + 32 * q, row = i0 + lane;
+            int mb, n0, ncols;
+            item_of<BN>(t, ntm, sym, nfull, mb, n0, ncols);
+            const int i0 = mb * kBM + 32 * q, row = i0 + lane;
             // first column block of this warp: in a symmetric product the
             // blocks left of the diagonal are skipped
             const int cfirst = sym ? max(0, i0 - n0) : 0;
             uint32_t dn[16];  // D of the next block, loaded one block ahead
             if (useD) load_d(dn, G, row, n0 + cfirst);
-            for (int c0 = cfirst; c0 < BN; c0 += 32) {
+            for (int c0 = cfirst; c0 < ncols; c0 += 32) {
                 const int col0 = n0 + c0;
                 uint32_t dc[16];
 #pragma unroll
                 for (int j = 0; j < 16; ++j) dc[j] = dn[j];
-                if (useD && c0 + 32 < BN) load_d(dn, G, row, col0 + 32);
+                if (useD && c0 + 32 < ncols) load_d(dn, G, row, col0 + 32);
                 float v[32];
                 tmem_ld32(tmem + static_cast<uint32_t>(b * BN + c0) + (static_cast<uint32_t>(32 * q) << 16), v);
                 if (useD) {
@@ -543,15 +572,21 @@ static_assert(sizeof(TcSmem<128>) + 1024 <= 232448 && sizeof(TcSmem<256>) + 1024
               "shared memory per CTA");
 
 template <int BN>
-cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorMap& mc, const CUtensorMap& mct,
-                      const GemmArgs& G, cudaStream_t st) {
+cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorMap& mbh, const CUtensorMap& mc,
+                      const CUtensorMap& mct, GemmArgs G, cudaStream_t st) {
     const int smem = static_cast<int>(sizeof(TcSmem<BN>)) + 1024;
     cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     const int ntm = (G.M + kBM - 1) / kBM, ntn = (G.N + BN - 1) / BN;
     const int ntiles = G.sym ? ntn * (ntn + 1) / 2 : ntm * ntn;
-    const int grid = std::min(ntiles, device_sm_count());
-    k_gemm_tc<BN><<<grid, kTcThreads, smem, st>>>(ma, mb, mc, mct, G);
+    const int sms = device_sm_count();
+    // a last wave that fills at most half the SMs runs as half tiles on
+    // twice as many (symmetric products keep whole tiles)
+    const int tail = ntiles % sms;
+    G.nfull = (!G.sym && ntiles > sms && tail > 0 && 2 * tail <= sms) ? ntiles - tail : ntiles;
+    const int nitems = G.nfull + 2 * (ntiles - G.nfull);
+    const int grid = std::min(nitems, sms);
+    k_gemm_tc<BN><<<grid, kTcThreads, smem, st>>>(ma, mb, mbh, mc, mct, G);
     return cudaGetLastError();
 }
 
@@ -566,8 +601,10 @@ cudaError_t gemm_bf16_nt(int M, int N, int K, float alpha, const void* A, int ld
         // (and for symmetric products) 128-wide ones
         const int64_t tiles256 = static_cast<int64_t>((M + kBM - 1) / kBM) * ((N + 255) / 256);
         const int bn = (sym || tiles256 < device_sm_count()) ? 128 : 256;
-        CUtensorMap ma, mb, mc{}, mct{};
-        if (!make_map(&ma, A, M, K, lda, kBM) || !make_map(&mb, B, N, K, ldb, bn)) return cudaErrorInvalidValue;
+        CUtensorMap ma, mb, mbh, mc{}, mct{};
+        if (!make_map(&ma, A, M, K, lda, kBM) || !make_map(&mb, B, N, K, ldb, bn) ||
+            !make_map(&mbh, B, N, K, ldb, bn / 2))
+            return cudaErrorInvalidValue;
         if (C != nullptr && !make_map(&mc, C, M, N, ldc, 0)) return cudaErrorInvalidValue;
         if (CT != nullptr && !make_map(&mct, CT, N, M, ldct, 0)) return cudaErrorInvalidValue;
         if (sym) mct = mc;  // the mirrored blocks go to C itself
@@ -585,7 +622,8 @@ cudaError_t gemm_bf16_nt(int M, int N, int K, float alpha, const void* A, int ld
         G.ldct = ldct;
         G.sym = sym ? 1 : 0;
         G.err = err;
-        return bn == 128 ? launch_tc<128>(ma, mb, mc, mct, G, st) : launch_tc<256>(ma, mb, mc, mct, G, st);
+        G.nfull = 0;  // set by the launch
+        return bn == 128 ? launch_tc<128>(ma, mb, mbh, mc, mct, G, st) : launch_tc<256>(ma, mb, mbh, mc, mct, G, st);
     }
     const dim3 grid((N + 63) / 64, (M + 63) / 64);
     k_gemm_simt<__nv_bfloat16><<<grid, 256, 0, st>>>(

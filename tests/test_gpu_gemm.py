@@ -6,7 +6,8 @@ element may round to the neighbouring bf16 value: within 2^-7 relative plus
 operand ring wraps), ragged M, N and K, the Newton-Schulz shapes of a
 2048 x 8192 matrix, the transposed output, and leading dimensions that TMA
 cannot address (the CUDA-core path: lda = 100, and ldc = 700 in the 300 x 700
-case)."""
+case).  A last wave of tiles that fills at most half the SMs runs as half
+tiles: 2048 x 8192 and 2904 x 4008 (256-wide tiles), 2048 x 1536 (128-wide)."""
 import pytest
 import torch
 
@@ -30,7 +31,7 @@ def _close(got, ref):
 
 @pytest.mark.parametrize("M,N,K", [(128, 256, 64), (256, 512, 1024), (296, 712, 200), (64, 64, 256),
                                    (2048, 2048, 8192), (2048, 8192, 2048), (96, 512, 96),
-                                   (2904, 4008, 328), (300, 700, 200)])
+                                   (2904, 4008, 328), (300, 700, 200), (2048, 1536, 256)])
 @pytest.mark.parametrize("with_d", [False, True])
 def test_gemm_matches_fp32_product(M, N, K, with_d):
     g = torch.Generator(device="cuda").manual_seed(M * 7 + N + K)
