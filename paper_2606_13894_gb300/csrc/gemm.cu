@@ -296,6 +296,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     tc_fence_after();
     const uint32_t tmem = sm.tmem;
     volatile int* abort = &sm.abort;
+    // Launched as a programmatic dependent of the previous kernel on the
+    // stream: everything above overlapped its end; the operands (and the
+    // buffers written) may be that kernel's, so wait for it to complete.
+    // Then let the next product start its own prologue.
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
     int issued = 0;  // thread 0: k-tiles whose loads were started
     if (threadIdx.x == 0) {
@@ -585,9 +591,19 @@ cudaError_t launch_tc(const CUtensorMap& ma, const CUtensorMap& mb, const CUtens
     const int tail = ntiles % sms;
     G.nfull = (!G.sym && ntiles > sms && tail > 0 && 2 * tail <= sms) ? ntiles - tail : ntiles;
     const int nitems = G.nfull + 2 * (ntiles - G.nfull);
-    const int grid = std::min(nitems, sms);
-    k_gemm_tc<BN><<<grid, kTcThreads, smem, st>>>(ma, mb, mbh, mc, mct, G);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(std::min(nitems, sms)));
+    cfg.blockDim = dim3(kTcThreads);
+    cfg.dynamicSmemBytes = static_cast<size_t>(smem);
+    cfg.stream = st;
+    // programmatic dependent launch: the prologue overlaps the previous kernel
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, k_gemm_tc<BN>, ma, mb, mbh, mc, mct, G);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t gemm_bf16_nt(int M, int N, int K, float alpha, const void* A, int lda, const void* B, int ldb,
