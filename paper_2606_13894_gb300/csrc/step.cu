@@ -827,12 +827,36 @@ __device__ __forceinline__ void stream_tile(Smem& sm, const Ptrs& P, const HP& h
         fac[1] = fac[0]; inv[1] = inv[0];
         fac[3] = fac[2]; inv[3] = inv[2];
     } else if ((p & (p - 1)) == 0) {
-        // p in {16, 32, 64, 128}: a block spans p/4 lanes of one group
-        const int lanes = p >> 2;
+        // p in {16, 32, 64, 128}: a block spans p/4 lanes of one group.
+        // Reduce-scatter over the four groups: the two halves of a span swap
+        // the sums of two groups (each keeps a pair), the quarters swap one
+        // more, and a butterfly over the remaining lanes completes the one
+        // group a lane keeps -- the pairs combine as in a butterfly per group,
+        // so the sums are the same.  The lane derives that block's factors
+        // once; each lane then gathers its four groups' factors.
+        const int lanes = p >> 2, oa = lanes >> 1, ob = lanes >> 2;
+        const bool hi = (lane & oa) != 0, lo = (lane & ob) != 0;
+        float k0 = hi ? g2[2] : g2[0], k1 = hi ? g2[3] : g2[1];
+        float q0 = hi ? mx[2] : mx[0], q1 = hi ? mx[3] : mx[1];
+        k0 += __shfl_xor_sync(0xffffffffu, hi ? g2[0] : g2[2], oa);
+        k1 += __shfl_xor_sync(0xffffffffu, hi ? g2[1] : g2[3], oa);
+        q0 = fmaxf(q0, __shfl_xor_sync(0xffffffffu, hi ? mx[0] : mx[2], oa));
+        q1 = fmaxf(q1, __shfl_xor_sync(0xffffffffu, hi ? mx[1] : mx[3], oa));
+        float s2 = (lo ? k1 : k0) + __shfl_xor_sync(0xffffffffu, lo ? k0 : k1, ob);
+        float sx = fmaxf(lo ? q1 : q0, __shfl_xor_sync(0xffffffffu, lo ? q0 : q1, ob));
+        butterfly(s2, sx, ob);
+        const int g = (hi ? 2 : 0) + (lo ? 1 : 0);  // the group this lane completed
+        const float vg = g == 0 ? r_v[0] : g == 1 ? r_v[1] : g == 2 ? r_v[2] : r_v[3];
+        const int bg = g == 0 ? blk[0] : g == 1 ? blk[1] : g == 2 ? blk[2] : blk[3];
+        const bool lg = g == 0 ? live[0] : g == 1 ? live[1] : g == 2 ? live[2] : live[3];
+        float f, iv;
+        finish(s2, sx, vg, ti.bo + bg, lg && (lane & (ob - 1)) == 0, f, iv);
+        const int base = lane & ~(oa | ob);
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-            butterfly(g2[j], mx[j], lanes);
-            finish(g2[j], mx[j], r_v[j], ti.bo + blk[j], live[j] && (lane & (lanes - 1)) == 0, fac[j], inv[j]);
+            const int src = base | ((j & 2) ? oa : 0) | ((j & 1) ? ob : 0);
+            fac[j] = __shfl_sync(0xffffffffu, f, src);
+            inv[j] = __shfl_sync(0xffffffffu, iv, src);
         }
     } else {
         // any other shape: each group's partial goes over the thread's own
