@@ -227,9 +227,13 @@ __device__ __forceinline__ uint32_t byte_of(uint4 c, int i) {
 }
 
 // ------------------------------------------------------------------ p == 1
-// Every element is its own block: v and s are per element, x = m/|m| = +-1.
-// With two codes per byte a thread owns both elements of a byte (a pair);
-// the nibble of an element past the tensor's end is left as it was.
+// Every element is its own block: v and s are per element, x = m/|m| = +-1,
+// so its level is one of two, found once per CTA (an infinite m gives x = NaN
+// and level 0, m = 0 the level of 0).  With two codes per byte a thread owns
+// both elements of a byte (a pair); the nibble of an element past the
+// tensor's end is left as it was.  fp32 theta and 8-bit codes whose blocks
+// start on a multiple of four take four elements per thread with 16-byte
+// accesses.
 template <int MODE, int FMT>
 __global__ void __launch_bounds__(kThreads) k_step_p1(const __grid_constant__ Launch L, const Ptrs P) {
     constexpr int EPC = Format<FMT>::kC4 ? 2 : 1;  // elements per thread and step
@@ -241,10 +245,59 @@ __global__ void __launch_bounds__(kThreads) k_step_p1(const __grid_constant__ La
     const int64_t base = (unit - S.unit_begin) * (4 * kThreads * EPC);
     const HP& hp = L.hp;
     const int zero_code = (MODE != kGradOnly) ? level_search(s_mid, 0.0f) : 0;
+    const int cpos = (MODE != kGradOnly) ? level_search(s_mid, 1.0f) : 0;
+    const int cneg = (MODE != kGradOnly) ? level_search(s_mid, -1.0f) : 0;
+    // the level of m (and x = m / |m| for the histogram)
+    auto level = [&](float m, float am, float& x) -> int {
+        if (am > 0.0f) {
+            x = __fdiv_rn(m, am);
+            return isinf(m) ? 0 : (m > 0.0f ? cpos : cneg);
+        }
+        x = __int_as_float(0x7fffffff);
+        return zero_code;
+    };
+    if (FMT == 0 && MODE != kGradOnly && ((S.block_off & 3) | (S.elem_off & 3)) == 0 &&
+        ((reinterpret_cast<uintptr_t>(P.v) | reinterpret_cast<uintptr_t>(P.scale)) & 15u) == 0) {
+        const int64_t le = base + 4 * static_cast<int64_t>(threadIdx.x);
+        if (le + 4 <= S.numel) {
+            const int64_t e = S.elem_off + le, bi = S.block_off + le;
+            const uint2 gw = __ldcs(reinterpret_cast<const uint2*>(P.grads + e));
+            const uint32_t cw = __ldcs(reinterpret_cast<const unsigned int*>(P.codes + e));
+            const float4 sc = *reinterpret_cast<const float4*>(P.scale + bi);
+            const float4 vv = *reinterpret_cast<const float4*>(P.v + bi);
+            const float4 tt = __ldcs(reinterpret_cast<const float4*>(P.params + e));
+            const float g[4] = {bf16_lo(gw.x), bf16_hi(gw.x), bf16_lo(gw.y), bf16_hi(gw.y)};
+            const float s4[4] = {sc.x, sc.y, sc.z, sc.w}, v4[4] = {vv.x, vv.y, vv.z, vv.w};
+            const float t4[4] = {tt.x, tt.y, tt.z, tt.w};
+            float mo[4], vo[4], to[4], xo[4];
+            uint32_t co = 0u;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const float m = fmaf(hp.omb1, g[q], hp.beta1 * s4[q] * s_dec[(cw >> (8 * q)) & 0xFFu]);
+                const float vn = fmaf(hp.beta2, v4[q], hp.omb2 * (g[q] * g[q]));
+                const float fac = hp.lr_bc1 / (sqrtf(vn * hp.inv_bc2) + hp.eps);
+                mo[q] = fabsf(m);
+                vo[q] = vn;
+                to[q] = fmaf(-fac, m, hp.decay * t4[q]);
+                co |= static_cast<uint32_t>(level(m, mo[q], xo[q])) << (8 * q);
+            }
+            *reinterpret_cast<float4*>(P.v + bi) = make_float4(vo[0], vo[1], vo[2], vo[3]);
+            *reinterpret_cast<float4*>(P.scale + bi) = make_float4(mo[0], mo[1], mo[2], mo[3]);
+            __stcs(reinterpret_cast<float4*>(P.params + e), make_float4(to[0], to[1], to[2], to[3]));
+            __stcs(reinterpret_cast<unsigned int*>(P.codes + e), co);
+            if (MODE == kHist) __stcs(reinterpret_cast<float4*>(P.xstage + e), make_float4(xo[0], xo[1], xo[2], xo[3]));
+            return;
+        }
+        if (le >= S.numel) return;
+        // the tensor's last one to three elements: the scalar form below, by this thread
+    }
+    const bool vec = FMT == 0 && MODE != kGradOnly && ((S.block_off & 3) | (S.elem_off & 3)) == 0 &&
+                     ((reinterpret_cast<uintptr_t>(P.v) | reinterpret_cast<uintptr_t>(P.scale)) & 15u) == 0;
     uint16_t* th16 = reinterpret_cast<uint16_t*>(P.params);
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-        const int64_t c0 = base + (threadIdx.x + i * kThreads) * static_cast<int64_t>(EPC);
+        const int64_t c0 = vec ? base + 4 * static_cast<int64_t>(threadIdx.x) + i
+                               : base + (threadIdx.x + i * kThreads) * static_cast<int64_t>(EPC);
         if (c0 >= S.numel) break;
         uint32_t cbyte = 0u;
         if (MODE != kGradOnly && Format<FMT>::kC4) cbyte = P.codes[(S.elem_off + c0) >> 1];
@@ -271,14 +324,7 @@ __global__ void __launch_bounds__(kThreads) k_step_p1(const __grid_constant__ La
             else
                 __stcs(P.params + e, tn);
             float x;
-            int c;
-            if (am > 0.0f) {
-                x = __fdiv_rn(m, am);
-                c = level_search(s_mid, x);
-            } else {
-                x = __int_as_float(0x7fffffff);
-                c = zero_code;
-            }
+            const int c = level(m, am, x);
             if (Format<FMT>::kC4)
                 cbyte = (cbyte & ~(0xFu << (4 * q))) | (static_cast<uint32_t>(c) << (4 * q));
             else

@@ -12,7 +12,9 @@ from paper_2606_13894_gb300 import gefen as G
 pytestmark = pytest.mark.gpu
 
 PATH_CASES = {
-    "p1": [(1000, 1), (4096, 1)],
+    # blocks of one: the first tensor four at a time (three left for the
+    # scalar form), the others at block offsets that are not multiples of four
+    "p1": [(999, 1), (4096, 1), (1000, 1)],
     "stream4k": [(64 * 300, 64), (2048 * 7, 2048), (4096 * 3, 4096), (16 * 999, 16), (768 * 5, 768), (48 * 401, 48)],
     "stream8k": [(8192 * 3, 8192), (6144 * 5, 6144), (4112 * 4, 4112)],
     "tile16_v4": [(16384 * 3, 16384), (12288 * 2, 12288)],
