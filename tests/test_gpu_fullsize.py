@@ -144,7 +144,7 @@ def test_gpt2_125m_set_sampled_parity():
 
 
 @pytest.mark.parametrize("log2n,p", [(20, 1), (20, 64), (20, 4096), (20, 1 << 20), (24, 4096), (26, 1 << 26),
-                                     (28, 64), (31, 4096), (31, 1 << 20)])
+                                     (28, 1), (28, 64), (31, 4096), (31, 1 << 20)])
 def test_flat_sweep_sampled_parity(log2n, p):
     n = 1 << log2n
     per = min(n // p, 256 if p <= 4096 else 2)  # blocks sampled (small blocks: many)
