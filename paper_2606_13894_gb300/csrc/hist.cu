@@ -4,15 +4,13 @@
 // HBM-bound: 4 bytes read per value.  Counts are privatised in shared memory
 // and flushed to the u64 result once per CTA.  Up to 16384 cells: u32
 // counters, two CTAs per SM.  Up to 65536 cells, one CTA per SM: u32 counters
-// for the (at most 49152) central cells, where normalised momentum piles up,
-// and two 16-bit counters per u32 word for the outer ones (224 KB at 65536
-// cells), kept below 2^16 by construction: after every kPackedUnits units (at
-// most 49152 values) the CTA moves each outer counter that has reached 2^14
-// to the u64 result, so between checks none can pass 2^14 - 1 + 49152 =
-// 65535.  That path computes a cell in seven instructions (a round-down add of
-// 1.5 * 2^23 takes the floor), lets a warp whose 512 values of a round share
-// one cell count them with a single atomic, and asks L2 for its next units
-// ahead of the loads.  NaN values are skipped.
+// for the (at most 57344) central cells, where normalised momentum piles up,
+// and for the kEdge cells at each end (every block's largest |x| is 1 and
+// lands there); the sparse shoulders between them are added straight to the
+// u64 result.  That path computes a cell in seven instructions (a round-down
+// add of 1.5 * 2^23 takes the floor), lets a warp whose 512 values of a round
+// share one cell count them with a single atomic, and asks L2 for its next
+// units ahead of the loads.  NaN values are skipped.
 #include <algorithm>
 #include <vector>
 
@@ -27,8 +25,6 @@ constexpr int kHistThreads = 1024;
 constexpr int kHistMaxRanges = 512;
 constexpr int64_t kHistUnit = 16384;  // values per work unit
 constexpr int kHistLoads = 4;         // float4 loads in flight per thread
-constexpr int kPackedUnits = 3;       // units between checks of the 16-bit counters
-constexpr unsigned kSpillAt = 1u << 14;
 
 struct HistLaunch {
     int32_t nranges;
@@ -105,14 +101,14 @@ __global__ void __launch_bounds__(kHistThreads) k_hist1(const float* __restrict_
     }
 }
 
-// ------------------------------------------------- 16-bit counter path
+// ------------------------------------------------- 65536-cell path
 // Cells of the 65536-cell path as the bits of a float: the floor of the cell
 // coordinate is taken by a round-down add of 1.5 * 2^23, so that the sum's
 // bits minus kMagicBits are the cell (coordinates below 2^22 here).  With B a
 // power of two the scaling by B/2 is exact, so RN(x + 1) * B/2 floored by one
 // round-down fma is the cell definition's floor(RN(RN(x + 1) * B/2)), clamped
 // in the integer domain; other B take the definition's two roundings, clamped
-// in fp32.  NaN maps to nan_bits (the trash counter, see Cells).
+// in fp32.  NaN maps to nan_bits (the caller's marker of a skipped value).
 constexpr float kMagic = 12582912.0f;  // 1.5 * 2^23
 constexpr uint32_t kMagicBits = 0x4B400000u;
 
@@ -129,67 +125,39 @@ __device__ __forceinline__ uint32_t cell_bits(float x, float halfB, float top, i
     return isnan(x) ? nan_bits : c;
 }
 
-// Counters of the 16384 < B <= 65536 path: the ncen central cells
-// [c_lo, c_lo + ncen) have u32 counters (ncen <= 49152: 192 KB); the at most
-// 16384 outer cells share u32 words two at a time as 16-bit counters (outer
-// index o: the cells below c_lo first, then those above the central run),
-// followed by one trash word that NaN values count into (never read).
-// Normalised momentum piles up near 0, so most counts go to u32 counters,
-// which need no overflow checks.
+// Counters of the 16384 < B <= 65536 path: u32 counters in shared memory for
+// the ncen central cells [c_lo, c_lo + ncen) and the `edge` cells at each end
+// ([0, edge) then [B - edge, B)); a cell between them is added to the u64
+// result directly.  Normalised momentum piles up near 0, and each block's
+// largest |x| is 1 (an end cell), so the cells left to global atomics hold
+// the few values between.
 struct Cells {
     unsigned* cen;
-    unsigned* outer;  // outer index o: half o & 1 of word o / 2; word nw: trash
-    uint32_t c_lo, ncen;
+    unsigned* ext;
+    uint32_t c_lo, ncen, edge, B;
 };
 
-constexpr uint32_t kMaxCentral = 49152;
+constexpr uint32_t kMaxCentral = 57344;  // 224 KB of u32 counters
+constexpr uint32_t kEdge = 32;
 
-// Adds n counts to cell (bits) c, without a branch.
-__device__ __forceinline__ void count_bits(const Cells& S, uint32_t c, unsigned n) {
-    const uint32_t ci = c - kMagicBits, d = ci - S.c_lo;
-    const bool cen = d < S.ncen;
-    const uint32_t o = ci < S.c_lo ? ci : ci - S.ncen;
-    unsigned* w = cen ? S.cen + d : S.outer + (o >> 1);
-    atomicAdd(w, cen ? n : n << ((o & 1u) << 4));
+__host__ __device__ constexpr uint32_t central_cells(uint32_t B) { return B < kMaxCentral ? B : kMaxCentral; }
+__host__ __device__ constexpr uint32_t edge_cells(uint32_t B) {
+    return (B - central_cells(B)) / 2 < kEdge ? (B - central_cells(B)) / 2 : kEdge;
 }
 
-// Cell of outer index o.
-__device__ __forceinline__ int outer_cell(const Cells& S, uint32_t o) {
-    return static_cast<int>(o < S.c_lo ? o : o + S.ncen);
-}
-
-// Moves every outer 16-bit counter that has reached kSpillAt to the u64
-// result; four words are tested at once and only words with a counter at or
-// above 2^14 are touched (between two CTA barriers: no count is in flight).
-__device__ __forceinline__ void spill_packed4(const Cells& S, int nw, uint64_t* __restrict__ hist) {
-    static_assert(kSpillAt == (1u << 14), "the test below looks at bits 14 and 15");
-    unsigned* words = S.outer;
-    auto one = [&](int i) {
-        const unsigned w = words[i];
-        const unsigned lo = w & 0xFFFFu, hi = w >> 16;
-        unsigned keep = w;
-        if (lo >= kSpillAt) {
-            atomicAdd(reinterpret_cast<unsigned long long*>(hist + outer_cell(S, 2 * i)),
-                      static_cast<unsigned long long>(lo));
-            keep &= 0xFFFF0000u;
-        }
-        if (hi >= kSpillAt) {
-            atomicAdd(reinterpret_cast<unsigned long long*>(hist + outer_cell(S, 2 * i + 1)),
-                      static_cast<unsigned long long>(hi));
-            keep &= 0x0000FFFFu;
-        }
-        if (keep != w) words[i] = keep;
-    };
-    const uint4* w4 = reinterpret_cast<const uint4*>(words);
-    for (int i = threadIdx.x; i < (nw >> 2); i += blockDim.x) {
-        const uint4 a = w4[i];
-        if (((a.x | a.y | a.z | a.w) & 0xC000C000u) == 0u) continue;
-        one(4 * i);
-        one(4 * i + 1);
-        one(4 * i + 2);
-        one(4 * i + 3);
+// Adds n counts to cell c (0xFFFFFFFF: a NaN value, skipped).
+__device__ __forceinline__ void count_cell(const Cells& S, uint64_t* __restrict__ hist, uint32_t c, unsigned n) {
+    const uint32_t d = c - S.c_lo;
+    if (d < S.ncen) {
+        atomicAdd(S.cen + d, n);
+    } else if (c < S.B) {
+        if (c < S.edge)
+            atomicAdd(S.ext + c, n);
+        else if (c >= S.B - S.edge)
+            atomicAdd(S.ext + S.edge + (c - (S.B - S.edge)), n);
+        else
+            atomicAdd(reinterpret_cast<unsigned long long*>(hist + c), static_cast<unsigned long long>(n));
     }
-    for (int i = (nw & ~3) + static_cast<int>(threadIdx.x); i < nw; i += blockDim.x) one(i);
 }
 
 // Asks L2 to fetch the 16-byte aligned body of unit u (no registers or
@@ -206,15 +174,13 @@ __device__ __forceinline__ void prefetch_unit_l2(const float* __restrict__ x, co
 
 constexpr int kPrefetchUnits = 2;  // units of this CTA ahead of the one it counts
 
-// 16384 < B <= 65536 cells (Cells: u32 central counters, 16-bit outer pairs;
-// 224 KB at 65536 cells, one CTA per SM).  Shared memory leaves room for no
-// second CTA, so the loads in flight come from L2: thread 0 asks L2 for this
-// CTA's unit kPrefetchUnits ahead while the CTA counts, and each thread keeps
-// four 16-byte loads in flight.  When all 512 values of a warp's round fall in
-// one cell (or are all NaN) the warp adds them with one atomic, else every
-// value is one atomic.  After every kPackedUnits units (at most 49152 values)
-// the CTA moves each outer counter that has reached 2^14 to the u64 result,
-// so none can pass 2^14 - 1 + 49152 = 65535 and carry into its neighbour.
+// 16384 < B <= 65536 cells (Cells: u32 counters for the central and end
+// cells, 224 KB at 65536 cells, one CTA per SM).  Shared memory leaves room
+// for no second CTA, so the loads in flight come from L2: thread 0 asks L2
+// for this CTA's unit kPrefetchUnits ahead while the CTA counts, and each
+// thread keeps four 16-byte loads in flight.  When all 512 values of a warp's
+// round fall in one cell (or are all NaN) the warp adds them with one atomic,
+// else every value is one atomic.
 template <bool POW2>
 __global__ void __launch_bounds__(kHistThreads, 1) k_hist16(const float* __restrict__ x,
                                                            const __grid_constant__ HistLaunch L,
@@ -222,14 +188,15 @@ __global__ void __launch_bounds__(kHistThreads, 1) k_hist16(const float* __restr
     extern __shared__ uint4 s_dyn[];
     const int B = L.bins;
     Cells S;
-    S.ncen = min(static_cast<uint32_t>(B), kMaxCentral);
-    S.c_lo = (static_cast<uint32_t>(B) - S.ncen) / 2;
+    S.B = static_cast<uint32_t>(B);
+    S.ncen = central_cells(S.B);
+    S.c_lo = (S.B - S.ncen) / 2;
+    S.edge = edge_cells(S.B);
     S.cen = reinterpret_cast<unsigned*>(s_dyn);
-    S.outer = S.cen + ((S.ncen + 3) & ~3u);  // 16-byte aligned for the four-word spill test
-    const int nw = static_cast<int>((static_cast<uint32_t>(B) - S.ncen + 1) >> 1);
-    for (int i = threadIdx.x; i < static_cast<int>((S.ncen + 3) & ~3u) + nw + 1; i += blockDim.x) S.cen[i] = 0u;
-    // NaN: outer index 2 nw, the low half of the trash word
-    const uint32_t nan_bits = kMagicBits + 2u * static_cast<uint32_t>(nw) + S.ncen;
+    S.ext = S.cen + S.ncen;
+    for (int i = threadIdx.x; i < static_cast<int>(S.ncen + 2 * S.edge); i += blockDim.x) S.cen[i] = 0u;
+    // a NaN value's cell bits: kMagicBits - 1, cell 0xFFFFFFFF
+    const uint32_t nan_bits = kMagicBits - 1u;
     const int top_bits = static_cast<int>(kMagicBits) + B - 1;
     if (threadIdx.x == 0)
         for (int p = 0; p < kPrefetchUnits; ++p) {
@@ -239,7 +206,7 @@ __global__ void __launch_bounds__(kHistThreads, 1) k_hist16(const float* __restr
     __syncthreads();
     const float halfB = 0.5f * static_cast<float>(B), top = static_cast<float>(B - 1);
     const int lane = threadIdx.x & 31;
-    int since = 0;  // units since the last check of the counters (uniform)
+    auto cell = [&](float v) { return cell_bits<POW2>(v, halfB, top, top_bits, nan_bits) - kMagicBits; };
     for (int64_t u = blockIdx.x; u < L.nunits; u += gridDim.x) {
         if (threadIdx.x == 0) {
             const int64_t un = u + static_cast<int64_t>(kPrefetchUnits) * gridDim.x;
@@ -252,10 +219,7 @@ __global__ void __launch_bounds__(kHistThreads, 1) k_hist16(const float* __restr
             // 16-byte aligned body with float4 loads; scalar head and tail
             int64_t h = (s0 + 3) & ~int64_t(3);
             if (h > s1) h = s1;
-            for (int64_t e = s0 + threadIdx.x; e < h; e += blockDim.x) {
-                const uint32_t c = cell_bits<POW2>(__ldcg(x + e), halfB, top, top_bits, nan_bits);
-                count_bits(S, c, 1u);
-            }
+            for (int64_t e = s0 + threadIdx.x; e < h; e += blockDim.x) count_cell(S, hist, cell(__ldcg(x + e)), 1u);
             const int64_t nv = (s1 - h) >> 2;
             const float4* xv = reinterpret_cast<const float4*>(x + h);
             for (int64_t jw = threadIdx.x & ~31; jw < nv; jw += kHistLoads * blockDim.x) {
@@ -268,32 +232,24 @@ __global__ void __launch_bounds__(kHistThreads, 1) k_hist16(const float* __restr
                 uint32_t c[4 * kHistLoads];
 #pragma unroll
                 for (int k = 0; k < kHistLoads; ++k) {
-                    c[4 * k] = cell_bits<POW2>(q[k].x, halfB, top, top_bits, nan_bits);
-                    c[4 * k + 1] = cell_bits<POW2>(q[k].y, halfB, top, top_bits, nan_bits);
-                    c[4 * k + 2] = cell_bits<POW2>(q[k].z, halfB, top, top_bits, nan_bits);
-                    c[4 * k + 3] = cell_bits<POW2>(q[k].w, halfB, top, top_bits, nan_bits);
+                    c[4 * k] = cell(q[k].x);
+                    c[4 * k + 1] = cell(q[k].y);
+                    c[4 * k + 2] = cell(q[k].z);
+                    c[4 * k + 3] = cell(q[k].w);
                 }
                 uint32_t diff = 0;
 #pragma unroll
                 for (int k = 1; k < 4 * kHistLoads; ++k) diff |= c[k] ^ c[0];
                 const uint32_t c0 = __shfl_sync(0xffffffffu, c[0], 0);
                 if (__all_sync(0xffffffffu, diff == 0u && c[0] == c0)) {
-                    if (lane == 0) count_bits(S, c0, 32u * 4u * kHistLoads);
+                    if (lane == 0) count_cell(S, hist, c0, 32u * 4u * kHistLoads);
                 } else {
 #pragma unroll
-                    for (int k = 0; k < 4 * kHistLoads; ++k) count_bits(S, c[k], 1u);
+                    for (int k = 0; k < 4 * kHistLoads; ++k) count_cell(S, hist, c[k], 1u);
                 }
             }
-            for (int64_t e = h + nv * 4 + threadIdx.x; e < s1; e += blockDim.x) {
-                const uint32_t c = cell_bits<POW2>(__ldcg(x + e), halfB, top, top_bits, nan_bits);
-                count_bits(S, c, 1u);
-            }
-        }
-        if (++since == kPackedUnits) {
-            since = 0;
-            __syncthreads();
-            spill_packed4(S, nw, hist);
-            __syncthreads();
+            for (int64_t e = h + nv * 4 + threadIdx.x; e < s1; e += blockDim.x)
+                count_cell(S, hist, cell(__ldcg(x + e)), 1u);
         }
     }
     __syncthreads();
@@ -301,15 +257,10 @@ __global__ void __launch_bounds__(kHistThreads, 1) k_hist16(const float* __restr
         const unsigned c = S.cen[i];
         if (c) atomicAdd(reinterpret_cast<unsigned long long*>(hist + S.c_lo + i), static_cast<unsigned long long>(c));
     }
-    const uint32_t nouter = static_cast<uint32_t>(B) - S.ncen;
-    for (int i = threadIdx.x; i < nw; i += blockDim.x) {
-        const unsigned w = S.outer[i];
-        const unsigned lo = w & 0xFFFFu, hi = w >> 16;
-        if (lo) atomicAdd(reinterpret_cast<unsigned long long*>(hist + outer_cell(S, 2 * i)),
-                          static_cast<unsigned long long>(lo));
-        if (hi && static_cast<uint32_t>(2 * i + 1) < nouter)
-            atomicAdd(reinterpret_cast<unsigned long long*>(hist + outer_cell(S, 2 * i + 1)),
-                      static_cast<unsigned long long>(hi));
+    for (int i = threadIdx.x; i < static_cast<int>(2 * S.edge); i += blockDim.x) {
+        const unsigned c = S.ext[i];
+        const uint32_t cl = i < static_cast<int>(S.edge) ? static_cast<uint32_t>(i) : S.B - 2 * S.edge + i;
+        if (c) atomicAdd(reinterpret_cast<unsigned long long*>(hist + cl), static_cast<unsigned long long>(c));
     }
 }
 
@@ -358,10 +309,9 @@ cudaError_t launch_histogram(const float* x, const HistRange* ranges, int nrange
             const int64_t grid = std::min<int64_t>(units, 2 * static_cast<int64_t>(sms));
             k_hist1<<<dim3(static_cast<unsigned>(grid)), kHistThreads, smem, stream>>>(x, L, hist);
         } else {
-            // u32 counters for up to 49152 central cells, 16-bit pairs for the
-            // rest, one trash word
-            const size_t ncen = std::min<size_t>(bins, 49152);
-            const size_t smem = ((ncen + 3) / 4 * 4 + (bins - ncen + 1) / 2 + 1) * sizeof(unsigned);
+            // u32 counters for the central cells and the cells at both ends
+            const uint32_t b32 = static_cast<uint32_t>(bins);
+            const size_t smem = static_cast<size_t>(central_cells(b32) + 2 * edge_cells(b32)) * sizeof(unsigned);
             const bool pow2 = (bins & (bins - 1)) == 0;
             auto k16 = pow2 ? k_hist16<true> : k_hist16<false>;
             e = cudaFuncSetAttribute(k16, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
