@@ -181,6 +181,29 @@ constexpr int kPrefetchUnits = 2;  // units of this CTA ahead of the one it coun
 // thread keeps four 16-byte loads in flight.  When all 512 values of a warp's
 // round fall in one cell (or are all NaN) the warp adds them with one atomic,
 // else every value is one atomic.
+// n counts for a value whose cell, before any clamp, is raw (see the kernel):
+// a central cell at once, the rest through count_cell.  With B a power of
+// two, raw >= B is a value outside [-1, 1) or NaN: raw + kMagicBits are the
+// bits of the round-down fma, which is NaN for NaN (skipped), below 1.5 *
+// 2^23 for x < -1 (cell 0) and above it for x >= 1 (cell B - 1), as the cell
+// definition clamps; other B pass the clamped cell, and raw >= B is NaN.
+template <bool POW2>
+__device__ __forceinline__ void count_raw(const Cells& S, uint64_t* __restrict__ hist, uint32_t raw, unsigned n) {
+    const uint32_t d = raw - S.c_lo;
+    if (d < S.ncen) {
+        atomicAdd(S.cen + d, n);
+        return;
+    }
+    uint32_t c = raw;
+    if (raw >= S.B) {
+        if (!POW2) return;
+        const float f = __uint_as_float(raw + kMagicBits);
+        if (isnan(f)) return;
+        c = f < kMagic ? 0u : S.B - 1;
+    }
+    count_cell(S, hist, c, n);
+}
+
 template <bool POW2>
 __global__ void __launch_bounds__(kHistThreads, 1) k_hist16(const float* __restrict__ x,
                                                            const __grid_constant__ HistLaunch L,
@@ -206,7 +229,13 @@ __global__ void __launch_bounds__(kHistThreads, 1) k_hist16(const float* __restr
     __syncthreads();
     const float halfB = 0.5f * static_cast<float>(B), top = static_cast<float>(B - 1);
     const int lane = threadIdx.x & 31;
-    auto cell = [&](float v) { return cell_bits<POW2>(v, halfB, top, top_bits, nan_bits) - kMagicBits; };
+    // B a power of two: the cell of x in [-1, 1) before any clamp, one add and
+    // one round-down fma (x >= 1, x < -1, infinities and NaN all give raw >= B
+    // and are settled by count_raw); other B: the clamped cell.
+    auto cell = [&](float v) -> uint32_t {
+        if (POW2) return __float_as_uint(__fmaf_rd(__fadd_rn(v, 1.0f), halfB, kMagic)) - kMagicBits;
+        return cell_bits<false>(v, halfB, top, top_bits, nan_bits) - kMagicBits;
+    };
     for (int64_t u = blockIdx.x; u < L.nunits; u += gridDim.x) {
         if (threadIdx.x == 0) {
             const int64_t un = u + static_cast<int64_t>(kPrefetchUnits) * gridDim.x;
@@ -219,7 +248,9 @@ __global__ void __launch_bounds__(kHistThreads, 1) k_hist16(const float* __restr
             // 16-byte aligned body with float4 loads; scalar head and tail
             int64_t h = (s0 + 3) & ~int64_t(3);
             if (h > s1) h = s1;
-            for (int64_t e = s0 + threadIdx.x; e < h; e += blockDim.x) count_cell(S, hist, cell(__ldcg(x + e)), 1u);
+            for (int64_t e = s0 + threadIdx.x; e < h; e += blockDim.x) {
+                count_raw<POW2>(S, hist, cell(__ldcg(x + e)), 1u);
+            }
             const int64_t nv = (s1 - h) >> 2;
             const float4* xv = reinterpret_cast<const float4*>(x + h);
             for (int64_t jw = threadIdx.x & ~31; jw < nv; jw += kHistLoads * blockDim.x) {
@@ -242,14 +273,16 @@ __global__ void __launch_bounds__(kHistThreads, 1) k_hist16(const float* __restr
                 for (int k = 1; k < 4 * kHistLoads; ++k) diff |= c[k] ^ c[0];
                 const uint32_t c0 = __shfl_sync(0xffffffffu, c[0], 0);
                 if (__all_sync(0xffffffffu, diff == 0u && c[0] == c0)) {
-                    if (lane == 0) count_cell(S, hist, c0, 32u * 4u * kHistLoads);
+                    // equal raw cells are one cell (or all NaN, or all clamped alike)
+                    if (lane == 0) count_raw<POW2>(S, hist, c0, 32u * 4u * kHistLoads);
                 } else {
 #pragma unroll
-                    for (int k = 0; k < 4 * kHistLoads; ++k) count_cell(S, hist, c[k], 1u);
+                    for (int k = 0; k < 4 * kHistLoads; ++k) count_raw<POW2>(S, hist, c[k], 1u);
                 }
             }
-            for (int64_t e = h + nv * 4 + threadIdx.x; e < s1; e += blockDim.x)
-                count_cell(S, hist, cell(__ldcg(x + e)), 1u);
+            for (int64_t e = h + nv * 4 + threadIdx.x; e < s1; e += blockDim.x) {
+                count_raw<POW2>(S, hist, cell(__ldcg(x + e)), 1u);
+            }
         }
     }
     __syncthreads();

@@ -24,8 +24,9 @@ def _refit_from_hist(h, k):
     return cbo.cpu().numpy(), cs.cpu().numpy(), float(cost.cpu()[0]), ke, ws
 
 
-# 16385 and 65535: the two CTAs of a cell-splitting pair own halves that
-# differ by one cell
+# 16385 and 65535: cell counts that are not powers of two (the clamped cell
+# form); 65536 and 65535: the kernel whose end cells and shoulders leave the
+# central shared-memory counters
 @pytest.mark.parametrize("bins", [16, 4096, 65536, 1000, 16385, 65535])
 @pytest.mark.parametrize("n", [0, 1, 7, 100_003, 3_000_001])
 def test_histogram_bit_exact(bins, n):
