@@ -187,13 +187,14 @@ constexpr int kPrefetchUnits = 2;  // units of this CTA ahead of the one it coun
 // bits of the round-down fma, which is NaN for NaN (skipped), below 1.5 *
 // 2^23 for x < -1 (cell 0) and above it for x >= 1 (cell B - 1), as the cell
 // definition clamps; other B pass the clamped cell, and raw >= B is NaN.
+// (The kernel passes d = raw - c_lo.)
 template <bool POW2>
-__device__ __forceinline__ void count_raw(const Cells& S, uint64_t* __restrict__ hist, uint32_t raw, unsigned n) {
-    const uint32_t d = raw - S.c_lo;
+__device__ __forceinline__ void count_raw(const Cells& S, uint64_t* __restrict__ hist, uint32_t d, unsigned n) {
     if (d < S.ncen) {
         atomicAdd(S.cen + d, n);
         return;
     }
+    const uint32_t raw = d + S.c_lo;
     uint32_t c = raw;
     if (raw >= S.B) {
         if (!POW2) return;
@@ -232,9 +233,11 @@ __global__ void __launch_bounds__(kHistThreads, 1) k_hist16(const float* __restr
     // B a power of two: the cell of x in [-1, 1) before any clamp, one add and
     // one round-down fma (x >= 1, x < -1, infinities and NaN all give raw >= B
     // and are settled by count_raw); other B: the clamped cell.
+    // (returned relative to the central run: raw - c_lo, one subtraction)
+    const uint32_t base_bits = kMagicBits + S.c_lo;
     auto cell = [&](float v) -> uint32_t {
-        if (POW2) return __float_as_uint(__fmaf_rd(__fadd_rn(v, 1.0f), halfB, kMagic)) - kMagicBits;
-        return cell_bits<false>(v, halfB, top, top_bits, nan_bits) - kMagicBits;
+        if (POW2) return __float_as_uint(__fmaf_rd(__fadd_rn(v, 1.0f), halfB, kMagic)) - base_bits;
+        return cell_bits<false>(v, halfB, top, top_bits, nan_bits) - base_bits;
     };
     for (int64_t u = blockIdx.x; u < L.nunits; u += gridDim.x) {
         if (threadIdx.x == 0) {
@@ -268,11 +271,17 @@ __global__ void __launch_bounds__(kHistThreads, 1) k_hist16(const float* __restr
                     c[4 * k + 2] = cell(q[k].z);
                     c[4 * k + 3] = cell(q[k].w);
                 }
-                uint32_t diff = 0;
-#pragma unroll
-                for (int k = 1; k < 4 * kHistLoads; ++k) diff |= c[k] ^ c[0];
+                // one cell for the whole round?  Three of each lane's values
+                // first (random data fails there), then all of them
                 const uint32_t c0 = __shfl_sync(0xffffffffu, c[0], 0);
-                if (__all_sync(0xffffffffu, diff == 0u && c[0] == c0)) {
+                bool one = __all_sync(0xffffffffu, c[0] == c0 && c[2 * kHistLoads] == c0 && c[4 * kHistLoads - 1] == c0);
+                if (one) {
+                    uint32_t diff = 0;
+#pragma unroll
+                    for (int k = 1; k < 4 * kHistLoads; ++k) diff |= c[k] ^ c0;
+                    one = __all_sync(0xffffffffu, diff == 0u);
+                }
+                if (one) {
                     // equal raw cells are one cell (or all NaN, or all clamped alike)
                     if (lane == 0) count_raw<POW2>(S, hist, c0, 32u * 4u * kHistLoads);
                 } else {
