@@ -521,22 +521,27 @@ def flat_sweep(G, synth, dev, stream, hbm, sizes=(1 << 28, 1 << 31)):
 def refit_microbench(G, synth, dev, n=MICRO_N, bins=MICRO_BINS):
     """Histogram of n normalised values (default 1.5e9) into `bins` cells
     (default 65536), then the exact DP to 256 levels; CUDA-event times of each
-    part (after one untimed run)."""
+    part (after one untimed run): the median of three runs of the whole refit
+    from the values and of three from the histogram (the DP alone)."""
     x = synth.refit_values(n, SEED + 7, device=dev)
     hist = torch.zeros(bins, dtype=torch.int64, device=dev)
     cb = torch.empty(K, dtype=torch.float32, device=dev)
     ws = G.workspace(G.gefen_refit_workspace_size(bins, K), dev)
     G.gefen_refit_codebook(bins=bins, k=K, codebook_out=cb, x=x, hist_out=hist, workspace_buf=ws)
     torch.cuda.synchronize()
-    e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
-    e[0].record()
-    G.gefen_refit_codebook(bins=bins, k=K, codebook_out=cb, x=x, hist_out=hist, workspace_buf=ws)
-    e[1].record()
-    G.gefen_refit_codebook(bins=bins, k=K, codebook_out=cb, hist_in=hist, workspace_buf=ws)
-    e[2].record()
-    torch.cuda.synchronize()
+    whole, dp = [], []
+    for _ in range(3):
+        e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+        e[0].record()
+        G.gefen_refit_codebook(bins=bins, k=K, codebook_out=cb, x=x, hist_out=hist, workspace_buf=ws)
+        e[1].record()
+        G.gefen_refit_codebook(bins=bins, k=K, codebook_out=cb, hist_in=hist, workspace_buf=ws)
+        e[2].record()
+        torch.cuda.synchronize()
+        whole.append(e[0].elapsed_time(e[1]))
+        dp.append(e[1].elapsed_time(e[2]))
     ke = G.gefen_refit_status(ws)
-    hist_dp_ms, dp_ms = e[0].elapsed_time(e[1]), e[1].elapsed_time(e[2])
+    hist_dp_ms, dp_ms = sorted(whole)[1], sorted(dp)[1]
     del x
     torch.cuda.empty_cache()
     return {"values": n, "bins": bins, "levels": K, "k_eff": ke,
