@@ -23,7 +23,7 @@ namespace {
 
 constexpr int kHistThreads = 1024;
 constexpr int kHistMaxRanges = 512;
-constexpr int64_t kHistUnit = 16384;  // values per work unit
+constexpr int64_t kHistUnit = 32768;  // values per work unit
 constexpr int kHistLoads = 4;         // float4 loads in flight per thread
 
 struct HistLaunch {

@@ -50,7 +50,7 @@ def test_histogram_bit_exact(bins, n):
 def test_histogram_one_cell(bins, offset):
     # every value in one cell (x = 0 and its neighbours within the cell), a
     # start past the array's first element, counts far above 2^16 per CTA
-    # (about eight 16384-value units per CTA, most of them added 512 at a time)
+    # (about four 32768-value units per CTA, most of them added 512 at a time)
     n = 20_000_003
     x = np.zeros(n + offset, np.float32)
     x[offset + 1::7] = np.float32(0.25 / bins)
