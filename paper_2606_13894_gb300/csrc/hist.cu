@@ -12,6 +12,7 @@
 // share one cell count them with a single atomic, and asks L2 for its next
 // units ahead of the loads.  NaN values are skipped.
 #include <algorithm>
+#include <mutex>
 #include <vector>
 
 #include "common.cuh"
@@ -316,6 +317,26 @@ cudaError_t prepare_histogram() {
     return e;
 }
 
+// Resident CTAs per SM of k16 with `smem` bytes of shared memory on the
+// current device (1 if the query fails), cached per (device, kernel, size).
+static int hist16_per_sm(void (*k16)(const float*, HistLaunch, uint64_t*), bool pow2, size_t smem) {
+    static std::mutex mu;
+    static std::vector<std::pair<std::pair<int, size_t>, int>> cache;  // ((device * 2 + pow2, smem), CTAs)
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+    const int key = 2 * dev + (pow2 ? 1 : 0);
+    std::lock_guard<std::mutex> g(mu);
+    for (const auto& kv : cache)
+        if (kv.first.first == key && kv.first.second == smem) return kv.second;
+    int n = 1;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k16, kHistThreads, smem) != cudaSuccess || n < 1) {
+        (void)cudaGetLastError();
+        n = 1;
+    }
+    cache.push_back({{key, smem}, n});
+    return n;
+}
+
 cudaError_t launch_histogram(const float* x, const HistRange* ranges, int nranges, int bins, uint64_t* hist,
                              cudaStream_t stream) {
     // One launch sees at most 2^36 values, so a CTA's u32 counters (it handles
@@ -358,17 +379,8 @@ cudaError_t launch_histogram(const float* x, const HistRange* ranges, int nrange
             auto k16 = pow2 ? k_hist16<true> : k_hist16<false>;
             e = cudaFuncSetAttribute(k16, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
             if (e != cudaSuccess) return e;
-            // resident CTAs per SM for this size (asked once per size)
-            static thread_local size_t fit_smem = 0;
-            static thread_local int per_sm = 1;
-            if (fit_smem != smem) {
-                if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k16, kHistThreads, smem) !=
-                        cudaSuccess || per_sm < 1) {
-                    (void)cudaGetLastError();
-                    per_sm = 1;
-                }
-                fit_smem = smem;
-            }
+            // resident CTAs per SM for this size, asked once per device and size
+            const int per_sm = hist16_per_sm(k16, pow2, smem);
             const int64_t grid = std::min<int64_t>(units, static_cast<int64_t>(per_sm) * sms);
             k16<<<dim3(static_cast<unsigned>(grid)), kHistThreads, smem, stream>>>(x, L, hist);
         }
