@@ -56,13 +56,14 @@ K = 256
 HP = dict(lr=1e-4, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=0.0)  # Appendix I, Llama
 SEED = 0
 PROFILE = os.path.join(ROOT, "profiles", "step_stream4k_llama1p5b.md")
-DOMINANT = "k_step_stream<4096> (blocks of p <= 4096, p % 16 == 0, p > 1)"
+DOMINANT = "k_step_stream<4096, shape 512-multiple> (blocks of p <= 4096, p % 512 == 0)"
 
 
 def dominant(p: int) -> bool:
-    """Tensors served by the streamed 4096-element tile kernel, the one that
-    carries most of the step's bytes on this workload."""
-    return p > 1 and p % 16 == 0 and p <= 4096
+    """Tensors served by the streamed 4096-element tile kernel's launch for
+    blocks of whole warps' slices, the one that carries most of the step's
+    bytes on this workload."""
+    return p % 512 == 0 and p <= 4096
 
 
 def peaks():
@@ -76,7 +77,7 @@ def peaks():
 
 def step_kernel_source_hash() -> str:
     h = hashlib.sha256()
-    for f in ("step.cu", "common.cuh"):
+    for f in ("step.cu", "step_kernels.cuh", "step_s4k.cu", "common.cuh"):
         with open(os.path.join(ROOT, "paper_2606_13894_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
@@ -181,10 +182,10 @@ def launches_per_call(periods, flags_hist: bool) -> int:
     for p in periods:
         if p == 1:
             cls.add("p1")
-        elif p % 16 == 0 and p <= 4096:
-            cls.add("s4k")
         elif p % 16 == 0 and p <= 8192:
-            cls.add("s8k")
+            # one launch per block shape of the streamed classes
+            shape = "w" if p % 512 == 0 else ("s" if p <= 256 and (p & (p - 1)) == 0 else "a")
+            cls.add(("s4k" if p <= 4096 else "s8k") + shape)
         elif p % 16 == 0 and p <= 16384:
             cls.add("t16v4")
         elif p <= 2048:
