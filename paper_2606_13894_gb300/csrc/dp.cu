@@ -760,11 +760,13 @@ __device__ __forceinline__ bool grid_barrier(const DpWs& W, uint32_t target, lon
     return *s_abort != 0;
 }
 
-// Rows 0..n-1 of one phase over the grid's warps: warp gw takes row gw, the
-// rest come from the phase's counter.
+// Rows 0..n-1 of one phase over the grid's warps: warp w of CTA c takes row
+// w G + c (a CTA's warps spread over the whole range of end positions, so
+// each SM holds wide and narrow searches alike), the rest come from the
+// phase's counter.
 template <class F>
 __device__ __forceinline__ void for_rows(int n, uint32_t* counter, int gw, int nwarps, int lane, F&& f) {
-    int i = gw;
+    int i = (gw % kDpWarps) * static_cast<int>(gridDim.x) + gw / kDpWarps;
     while (i < n) {
         f(i);
         if (nwarps >= n) break;
