@@ -172,27 +172,35 @@ def dist_env():
     return ws, rank, local
 
 
-def launches_per_call(periods, flags_hist: bool) -> int:
-    """Kernels one gefen_step call launches for these periods (mirrors the
-    library's path classes; fewer than 300 tensors per class)."""
-    if not periods:
+SHAPE_SPLIT_ELEMS = 1 << 28  # the library's kShapeSplitElems
+
+
+def launches_per_call(entries, flags_hist: bool) -> int:
+    """Kernels one gefen_step call launches for these (period, numel) pairs
+    (mirrors the library's path classes; fewer than 300 tensors per class)."""
+    if not entries:
         return 0
-    cls = set()
+    classes = set()
     big = 0
-    for p in periods:
+    streamed = {}  # streamed class -> [elements, block shapes]
+    for p, n in entries:
         if p == 1:
-            cls.add("p1")
+            classes.add("p1")
         elif p % 16 == 0 and p <= 8192:
-            # one launch per block shape of the streamed classes
             shape = "w" if p % 512 == 0 else ("s" if p <= 256 and (p & (p - 1)) == 0 else "a")
-            cls.add(("s4k" if p <= 4096 else "s8k") + shape)
+            acc = streamed.setdefault("s4k" if p <= 4096 else "s8k", [0, set()])
+            acc[0] += n
+            acc[1].add(shape)
         elif p % 16 == 0 and p <= 16384:
-            cls.add("t16v4")
+            classes.add("t16v4")
         elif p <= 2048:
-            cls.add("gen")
+            classes.add("gen")
         else:
             big |= 1 if p % 16 == 0 else 2
-    n = len(cls) + 3 * bin(big).count("1")
+    # a streamed class launches once per block shape, or once in all when it
+    # has under SHAPE_SPLIT_ELEMS elements
+    n_streamed = sum(1 if tot < SHAPE_SPLIT_ELEMS else len(shapes) for tot, shapes in streamed.values())
+    n = len(classes) + n_streamed + 3 * bin(big).count("1")
     return n + (1 if flags_hist else 0)
 
 
@@ -390,7 +398,7 @@ def run_gpu(args, world, rank, local):
 
     e2e = run_e2e(G, cad, args, stream)
 
-    per = [[e[2] for e in ce] for ce in sh.call_entries]
+    per = [[(e[2], e[1]) for e in ce] for ce in sh.call_entries]
     n_launch_plain = sum(launches_per_call(x, False) for x in per)
     # refit steps: the step's calls with their histograms, then the DP's four
     # launches (prefix, first level, the cooperative levels launch, backtrack)

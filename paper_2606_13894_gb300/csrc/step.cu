@@ -763,12 +763,27 @@ cudaError_t launch_class(K kernel, Launch& L, const std::vector<int>& ids, const
     return cudaSuccess;
 }
 
+// Below this many elements a streamed class takes a single launch: a second
+// launch's fixed cost (table build, ramp and tail, about 10 us) exceeds what
+// a shape's own instance saves.
+constexpr int64_t kShapeSplitElems = int64_t(1) << 28;
+
 // The streamed kernel over the tensors `ids` of class c (kS4K or kS8K): one
-// launch (per segment-table group) for each block shape among them.
+// launch (per segment-table group) for each block shape among them, or one
+// launch in all for a class of under kShapeSplitElems elements (its shape's
+// instance when the shapes agree, else the instance for any shape).
 cudaError_t launch_stream(Launch& L, const std::vector<int>& ids, const gefen_tensor_t* t, PathClass c, int mode,
                           int hb, int fmt, const Ptrs& P, int* err, cudaStream_t st) {
     std::vector<int> by[3];
+    int64_t total = 0;
+    for (int id : ids) total += t[id].numel;
     for (int id : ids) by[shape_of(t[id].period)].push_back(id);
+    if (total < kShapeSplitElems && (by[0].size() != ids.size() && by[1].size() != ids.size() &&
+                                     by[2].size() != ids.size())) {
+        by[kShapeAny] = ids;
+        by[kShapeWarp].clear();
+        by[kShapeSub].clear();
+    }
     const int64_t cap = (c == kS4K) ? kS4KTile : kS8KTile;
     for (int shape : {kShapeWarp, kShapeSub, kShapeAny}) {
         cudaError_t e2 = cudaSuccess;
