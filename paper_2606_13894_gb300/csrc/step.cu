@@ -15,8 +15,7 @@
 //                                          whole blocks through shared memory
 //                                          (bulk copies): one HBM pass
 //                                          (step_kernels.cuh; one launch per
-//                                          block shape, or one for a class
-//                                          of under 2^28 elements)
+//                                          block shape)
 //   p % 16 == 0, p <= 16K  k_step_tile16   one CTA holds whole blocks in
 //                                          registers: one HBM pass
 //   other p <= 2048        k_step_generic  the same with scalar accesses
