@@ -486,7 +486,11 @@ __device__ __forceinline__ Best warp_min_best(Best b) {
     return Best{(static_cast<uint64_t>(hm) << 32) | lm, static_cast<int>(l)};
 }
 
-constexpr int kDpWarps = 16;     // warps (end positions at a time) per CTA
+// Warps (end positions at a time) per CTA of the levels kernel: 16 up to
+// kDpSmallBins cells (every row has its own warp), 8 above (anchored levels:
+// smaller CTAs wait at their block barrier for fewer rows; 65536 x 256 26.8
+// -> 26.1 ms, while 4096 x 256 took 2.92 ms against 2.83 with 16).
+constexpr int kDpWarpsSmall = 16, kDpWarpsLarge = 8, kDpSmallBins = 8192;
 constexpr int kStackCap = 192;   // runs pending per warp
 
 // Everything one warp needs to screen and evaluate candidates for one r.
@@ -764,9 +768,9 @@ __device__ __forceinline__ bool grid_barrier(const DpWs& W, uint32_t target, lon
 // w G + c (a CTA's warps spread over the whole range of end positions, so
 // each SM holds wide and narrow searches alike), the rest come from the
 // phase's counter.
-template <class F>
+template <int WARPS, class F>
 __device__ __forceinline__ void for_rows(int n, uint32_t* counter, int gw, int nwarps, int lane, F&& f) {
-    int i = (gw % kDpWarps) * static_cast<int>(gridDim.x) + gw / kDpWarps;
+    int i = (gw % WARPS) * static_cast<int>(gridDim.x) + gw / WARPS;
     while (i < n) {
         f(i);
         if (nwarps >= n) break;
@@ -780,15 +784,16 @@ __device__ __forceinline__ void for_rows(int n, uint32_t* counter, int gw, int n
 // between levels.  With anchors (P.stride > 0, interior levels), a level runs
 // in two phases: the anchor rows r = 0, stride, 2 stride, ... and b, then
 // (after a barrier) every other row, bracketed by its two anchors.
-__global__ void __launch_bounds__(kDpWarps * 32) k_dp_levels(DpLaunch P, DpWs W) {
-    __shared__ int2 s_stack[kDpWarps][kStackCap];
+template <int WARPS>
+__global__ void __launch_bounds__(WARPS * 32) k_dp_levels(DpLaunch P, DpWs W) {
+    __shared__ int2 s_stack[WARPS][kStackCap];
     __shared__ int s_abort;
     const Header h = *W.hdr;
     if (h.status) return;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t G = gridDim.x;
-    const int nwarps = static_cast<int>(G) * kDpWarps;
-    const int gw = static_cast<int>(blockIdx.x) * kDpWarps + warp;
+    const int nwarps = static_cast<int>(G) * WARPS;
+    const int gw = static_cast<int>(blockIdx.x) * WARPS + warp;
     const int B = P.B, S = P.stride;
     int2* stack = s_stack[warp];
     uint32_t nbar = 0;
@@ -796,15 +801,15 @@ __global__ void __launch_bounds__(kDpWarps * 32) k_dp_levels(DpLaunch P, DpWs W)
         uint32_t* ctr = W.sync + 1 + 3 * kk;
         if (S > 0 && kk < h.k_eff && h.b > S) {
             const int nA = h.b / S + 1 + (h.b % S ? 1 : 0);
-            for_rows(nA, ctr + 1, gw, nwarps, lane,
+            for_rows<WARPS>(nA, ctr + 1, gw, nwarps, lane,
                      [&](int i) { level_row(B, kk, min(i * S, h.b), S, kRowAnchor, W, h, lane, stack); });
             if (grid_barrier(W, ++nbar * G + P.barrier_extra, P.spin, &s_abort)) return;
-            for_rows(B + 1, ctr + 2, gw, nwarps, lane, [&](int r) {
+            for_rows<WARPS>(B + 1, ctr + 2, gw, nwarps, lane, [&](int r) {
                 if (r <= h.b && (r % S == 0 || r == h.b)) return;  // an anchor
                 level_row(B, kk, r, S, kRowBracket, W, h, lane, stack);
             });
         } else {
-            for_rows(B + 1, ctr, gw, nwarps, lane,
+            for_rows<WARPS>(B + 1, ctr, gw, nwarps, lane,
                      [&](int r) { level_row(B, kk, r, S, kRowFull, W, h, lane, stack); });
         }
         if (kk == P.k) break;
@@ -889,7 +894,8 @@ std::atomic<int> g_dbg_stride{-1};
 std::atomic<uint32_t> g_dbg_barrier_extra{0};
 std::atomic<long long> g_dbg_spin{0};
 
-// Resident CTAs per SM of k_dp_levels, asked once per device.
+// Resident CTAs per SM of k_dp_levels<WARPS>, asked once per device.
+template <int WARPS>
 int dp_levels_per_sm() {
     static std::mutex mu;
     static int cached[64] = {0};
@@ -898,13 +904,37 @@ int dp_levels_per_sm() {
     std::lock_guard<std::mutex> g(mu);
     if (cached[dev] == 0) {
         int n = 0;
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_dp_levels, kDpWarps * 32, 0) != cudaSuccess) {
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_dp_levels<WARPS>, WARPS * 32, 0) != cudaSuccess) {
             (void)cudaGetLastError();
             return 0;
         }
         cached[dev] = n;
     }
     return cached[dev];
+}
+
+// Levels 2..k: one cooperative launch of k_dp_levels<WARPS>.
+template <int WARPS>
+cudaError_t launch_levels(int bins, int k, const DpWs& W, cudaStream_t st) {
+    const int per_sm = dp_levels_per_sm<WARPS>();
+    if (per_sm < 1) return cudaErrorLaunchFailure;
+    const int rows = (bins + 1 + WARPS - 1) / WARPS;  // CTAs with a row each
+    const int grid = std::max(1, std::min(per_sm * device_sm_count(), rows));
+    DpLaunch P;
+    P.B = bins;
+    P.k = k;
+    // anchors pay off once the rows outnumber the grid's warps: each warp
+    // then searches one anchor row in full and brackets the rest
+    const int auto_stride = (bins + 1 > 2 * grid * WARPS) ? kAnchorStride : 0;
+    const int forced = g_dbg_stride.load();
+    P.stride = forced >= 0 ? forced : auto_stride;
+    P.barrier_extra = g_dbg_barrier_extra.load();
+    const long long spin = g_dbg_spin.load();
+    P.spin = spin > 0 ? spin : kBarrierSpin;
+    DpWs w = W;
+    void* args[] = {&P, &w};
+    return cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(k_dp_levels<WARPS>), dim3(grid), dim3(WARPS * 32),
+                                       args, 0, st);
 }
 
 }  // namespace
@@ -947,28 +977,9 @@ extern "C" gefen_status_t gefen_refit_codebook(const float* x, int64_t n, const 
     k_dp_prefix<<<1, kPrefixThreads, 0, st>>>(h, bins, k, W);
     const int grid1 = (bins + 2 + kDpThreads - 1) / kDpThreads;
     k_dp_level1<<<grid1, kDpThreads, 0, st>>>(bins, W);
-    {
-        const int per_sm = dp_levels_per_sm();
-        if (per_sm < 1) return GEFEN_ECUDA;
-        const int rows = (bins + 1 + kDpWarps - 1) / kDpWarps;  // CTAs with a row each
-        const int grid = std::max(1, std::min(per_sm * device_sm_count(), rows));
-        DpLaunch P;
-        P.B = bins;
-        P.k = k;
-        // anchors pay off once the rows outnumber the grid's warps: each warp
-        // then searches one anchor row in full and brackets the rest
-        const int auto_stride = (bins + 1 > 2 * grid * kDpWarps) ? kAnchorStride : 0;
-        const int forced = g_dbg_stride.load();
-        P.stride = forced >= 0 ? forced : auto_stride;
-        P.barrier_extra = g_dbg_barrier_extra.load();
-        const long long spin = g_dbg_spin.load();
-        P.spin = spin > 0 ? spin : kBarrierSpin;
-        DpWs w = W;
-        void* args[] = {&P, &w};
-        if (cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(k_dp_levels), dim3(grid), dim3(kDpWarps * 32),
-                                        args, 0, st) != cudaSuccess)
-            return GEFEN_ECUDA;
-    }
+    const cudaError_t el = (bins > kDpSmallBins) ? launch_levels<kDpWarpsLarge>(bins, k, W, st)
+                                                 : launch_levels<kDpWarpsSmall>(bins, k, W, st);
+    if (el != cudaSuccess) return GEFEN_ECUDA;
     k_dp_backtrack<<<1, 256, 0, st>>>(bins, k, W, codebook_out, cell_start_out, cost_out);
     if (cudaGetLastError() != cudaSuccess) return GEFEN_ECUDA;
     return GEFEN_OK;
@@ -1035,8 +1046,10 @@ gefen_status_t static_scratch(void** out) {
         cudaFuncAttributes fa;
         if (cudaFuncGetAttributes(&fa, k_dp_prefix) != cudaSuccess ||
             cudaFuncGetAttributes(&fa, k_dp_level1) != cudaSuccess ||
-            cudaFuncGetAttributes(&fa, k_dp_levels) != cudaSuccess ||
-            cudaFuncGetAttributes(&fa, k_dp_backtrack) != cudaSuccess || dp_levels_per_sm() < 1 ||
+            cudaFuncGetAttributes(&fa, k_dp_levels<kDpWarpsSmall>) != cudaSuccess ||
+            cudaFuncGetAttributes(&fa, k_dp_levels<kDpWarpsLarge>) != cudaSuccess ||
+            cudaFuncGetAttributes(&fa, k_dp_backtrack) != cudaSuccess || dp_levels_per_sm<kDpWarpsSmall>() < 1 ||
+            dp_levels_per_sm<kDpWarpsLarge>() < 1 ||
             prepare_histogram() != cudaSuccess) {
             (void)cudaGetLastError();
             return GEFEN_ECUDA;
