@@ -69,3 +69,26 @@ def test_reference_arm_under_torchrun_prints_one_line_from_rank_0():
     d = json.loads(lines[0])
     assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["value"] > 0
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["cpu_baseline"]["kind"] == "oracle"
+
+
+def test_launch_count_follows_the_librarys_launch_plan():
+    # The bench's gpu_launches claim mirrors gefen_step's plan: one launch
+    # per class of blocks; the streamed classes (p % 16 == 0, p <= 8192) once
+    # per block shape (multiples of 512; powers of two 16..256; any other),
+    # or once in all for a class of under 2^28 elements; three launches for
+    # big blocks (partial, finalise, apply); one more for a histogram step.
+    big = 1 << 28
+    # the Llama-shaped dominant call: blocks of 2048 and 512 share a shape
+    assert bench.launches_per_call([(2048, 934_805_504), (512, 8192)], False) == 1
+    # its second call: p = 1, 8192 tiles, blocks of 64 to 256, big blocks
+    second = [(1, 63_488), (8192, 335_544_320), (64, 75_499_520), (128, 8_392_704), (256, 6144),
+              (131072, 118_489_088), (262144, 6_291_456)]
+    assert bench.launches_per_call(second, False) == 1 + 1 + 1 + 3
+    assert bench.launches_per_call(second, True) == 7
+    # a large class of mixed shapes: one launch per shape
+    assert bench.launches_per_call([(2048, big), (64, big), (48, big)], False) == 3
+    # a small class of mixed shapes (the GPT-2-shaped set): one launch in all
+    assert bench.launches_per_call([(64, 75_108_096), (128, 46_857_216), (192, 2_361_600)], False) == 1
+    # other classes: 16K tiles, the generic tile, unaligned big blocks
+    assert bench.launches_per_call([(12288, 24576), (24, 4608), (30001, 60002)], False) == 1 + 1 + 3
+    assert bench.launches_per_call([], True) == 0
