@@ -106,13 +106,15 @@ struct StreamCfg {
 using S4KCfg = StreamCfg<4096, 256, 3, 8, 8, false, 2>;
 using S8KCfg = StreamCfg<8192, 512, 2, 8, 32, true, 1>;
 // Steps that also histogram x (refit steps) count up to kFusedBins cells in
-// shared memory.  To make room, the 4096 tiles' tables give up copies, and
-// the 8192 tiles read theta from global memory (an L2 hit after the issuing
-// thread's prefetch) instead of staging it: 8 copies of each table fit then,
-// and a refit step's 8192 tiles ran 6% faster than with theta staged and the
-// tables in 2 and 4 copies.
+// shared memory.  To make room, the 4096 tiles run two stages and keep the
+// decode table in 4 copies (the cell records keep 8: a refit step 2% faster
+// than with three stages and the records in 4), and the 8192 tiles read
+// theta from global memory (an L2 hit after the issuing thread's prefetch)
+// instead of staging it: 8 copies of each table fit then, and a refit step's
+// 8192 tiles ran 6% faster than with theta staged and the tables in 2 and 4
+// copies.
 constexpr int kFusedBins = 4096;
-using S4KHistCfg = StreamCfg<4096, 256, 3, 4, 8, false, 2>;
+using S4KHistCfg = StreamCfg<4096, 256, 2, 8, 4, false, 2>;
 using S8KHistCfg = StreamCfg<8192, 512, 2, 8, 8, false, 1>;
 constexpr int kS4KTile = S4KCfg::TILE, kS8KTile = S8KCfg::TILE;
 
