@@ -456,9 +456,10 @@ def run_gpu(args, world, rank, local):
 
 
 def cadence_65536(G, cad, args, stream, dev, nparams):
-    """The same job with refits from 65536-cell histograms (SURVEY's reading
-    for this set): the x of every tensor is staged and counted by the
-    65536-cell histogram kernel, then the 65536 x 256 DP."""
+    """The same job with refits from 65536-cell histograms (the other reading
+    of Algorithm 3's histogram size for this set: 65536 cells rather than 16
+    per level): the x of every tensor is staged and counted by the 65536-cell
+    histogram kernel, then the 65536 x 256 DP."""
     sh = cad.sh
     sh.set_refit_bins(65536)
     cad.reset_events()
